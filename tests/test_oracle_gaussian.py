@@ -1,0 +1,90 @@
+"""Pins for the oracle's Gaussian noise (Philox + Box-Muller, keyed by (seed, g)).
+
+Statistical checks use 5- to 6-sigma bands on fixed seeds, so a correct
+generator passes deterministically while a dropped factor (-2 ln u -> -ln u),
+a halved angle (pi u instead of 2 pi u), a reused uniform or a wrong lane/pair
+mapping fails one of them.
+"""
+import numpy as np
+from scipy import stats
+
+N_DRAWS = 1 << 22
+
+
+def _draws(oracle, seed, n=N_DRAWS, base=0):
+    return oracle.noise_fill(seed, base, n)
+
+
+def test_moments_per_lane(oracle):
+    x = _draws(oracle, 3)
+    lanes = x.reshape(-1, 4)
+    n = lanes.shape[0]
+    for k in range(4):
+        v = lanes[:, k]
+        assert abs(v.mean()) < 5 / np.sqrt(n), k
+        assert abs(v.var() - 1.0) < 5 * np.sqrt(2.0 / n), k
+        kurt = np.mean(v**4) / np.mean(v**2) ** 2
+        assert abs(kurt - 3.0) < 5 * np.sqrt(24.0 / n), k
+        assert abs(stats.skew(v)) < 5 * np.sqrt(6.0 / n), k
+
+
+def test_kolmogorov_smirnov_against_normal(oracle):
+    x = _draws(oracle, 11, n=1 << 20)
+    assert stats.kstest(x, "norm").pvalue > 1e-4
+    # the four lanes separately
+    for k in range(4):
+        assert stats.kstest(x[k::4], "norm").pvalue > 1e-4
+
+
+def test_lanes_seeds_and_blocks_uncorrelated(oracle):
+    n = 1 << 20
+    a = _draws(oracle, 5, n)
+    b = _draws(oracle, 6, n)          # neighbouring seed
+    lanes = a.reshape(-1, 4)
+    m = lanes.shape[0]
+    band = 6 / np.sqrt(m)
+    for i in range(4):
+        for j in range(i + 1, 4):
+            assert abs(np.corrcoef(lanes[:, i], lanes[:, j])[0, 1]) < band
+            # squares too: catches lanes that share a uniform
+            assert abs(np.corrcoef(lanes[:, i]**2, lanes[:, j]**2)[0, 1]) < band
+    assert abs(np.corrcoef(a, b)[0, 1]) < 6 / np.sqrt(n)
+    assert abs(np.corrcoef(a[:-4], a[4:])[0, 1]) < 6 / np.sqrt(n)   # adjacent blocks
+    assert abs(np.corrcoef(a**2, b**2)[0, 1]) < 6 / np.sqrt(n)
+
+
+def test_box_muller_pair_closed_form(oracle):
+    # Elements 4j and 4j+1 share a radius: eps0^2 + eps1^2 = -2 ln u(x0), and
+    # elements 4j+2, 4j+3 use x2: this pins which output word feeds which lane.
+    for seed, j in [(1, 0), (77, 12345), (2**40 + 3, 2**33)]:
+        x = oracle.noise_block(seed, j)
+        e = [oracle.gaussian(seed, 4 * j + k) for k in range(4)]
+        r01 = -2.0 * np.log(oracle.uniform(int(x[0])))
+        r23 = -2.0 * np.log(oracle.uniform(int(x[2])))
+        assert np.isclose(e[0] ** 2 + e[1] ** 2, r01, rtol=1e-13, atol=0)
+        assert np.isclose(e[2] ** 2 + e[3] ** 2, r23, rtol=1e-13, atol=0)
+        phi01 = np.arctan2(e[1], e[0]) % (2 * np.pi)
+        phi23 = np.arctan2(e[3], e[2]) % (2 * np.pi)
+        assert np.isclose(phi01, 2 * np.pi * oracle.uniform(int(x[1])), atol=1e-12)
+        assert np.isclose(phi23, 2 * np.pi * oracle.uniform(int(x[3])), atol=1e-12)
+
+
+def test_max_magnitude_bound(oracle):
+    # |eps| <= sqrt(-2 ln 2^-24) because u >= 2^-24.
+    bound = np.sqrt(-2.0 * np.log(2.0**-24))
+    x = _draws(oracle, 9, n=1 << 20)
+    assert np.max(np.abs(x)) <= bound
+    assert 5.768 < bound < 5.7682
+
+
+def test_noise_is_a_function_of_seed_and_index_only(oracle):
+    # The value at g does not depend on which range is filled (counter-based).
+    full = oracle.noise_fill(42, 1000, 64)
+    for off in (0, 3, 17, 63):
+        assert oracle.noise_fill(42, 1000 + off, 1)[0] == full[off]
+    g = np.array([1063, 1000, 1031], dtype=np.uint64)
+    assert np.array_equal(oracle.noise_at(42, g), full[[63, 0, 31]])
+    # and straddling the 2^32 block boundary of the 64-bit counter
+    base = 4 * 2**32 - 6
+    seg = oracle.noise_fill(8, base, 12)
+    assert np.array_equal(seg, oracle.noise_at(8, np.arange(base, base + 12, dtype=np.uint64)))
