@@ -1,0 +1,417 @@
+"""Throughput of the ES step on one GB300: param*seed/s of a full generation
+(N perturb + N restore + reward normalisation + one fused N-seed update) on a
+synthetic parameter set shaped like the paper's workloads.
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--workload qwen27b]
+                    [--impl ours|reference] [--no-e2e] [--no-cpu-baseline]
+
+Prints one JSON line (rank 0). `value` is measured with the inputs resident in
+HBM; `e2e` is the same metric with the parameters in pinned host memory and
+copied to the device and back inside every timed step. The reference arm
+(`--impl reference`) times the CPU oracle on a bounded sample of the same
+workload. With --gpus N > 1 (under torchrun) every rank runs an independent
+replica of the step (replicas only: the ES step has no exchange between GPUs
+besides N scalar rewards) and the slowest rank's time is reported.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+from paper_2608_17310_gb300 import inputs as I  # noqa: E402
+
+METRIC = "ES step param*seed/s (perturb+restore+update) and % of HBM/ALU roofline"
+UNIT = "param*seed/s"
+SIGMA_FINAL = {"qwen27b": 2.5e-4, "qwen4b": 5e-4, "toy": 1e-3}
+SCHEDULE_T = 100
+CPU_SAMPLE = 1 << 21
+
+
+def parse():
+    p = argparse.ArgumentParser()
+    p.add_argument("--gpus", type=int, default=1)
+    p.add_argument("--steps", type=int, default=5)
+    p.add_argument("--warmup", type=int, default=3)
+    p.add_argument("--workload", default="qwen27b", choices=["qwen27b", "qwen4b", "toy"])
+    p.add_argument("--population", type=int, default=None, help="override N")
+    p.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    p.add_argument("--no-e2e", action="store_true")
+    p.add_argument("--no-cpu-baseline", action="store_true")
+    p.add_argument("--e2e-steps", type=int, default=2)
+    return p.parse_args()
+
+
+def peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(path):
+        with open(path) as f:
+            d = json.load(f)
+        return float(d["hbm_gbs"]), float(d.get("sm_max_mhz", 2070.0)), "measured"
+    return 6800.0, 2070.0, "fallback"
+
+
+# --- distributed plumbing -------------------------------------------------------------
+
+def dist_setup(args):
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    if world == 1:
+        return 0, 1, None
+    import torch
+    import torch.distributed as dist
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    backend = "nccl" if torch.cuda.is_available() else "gloo"
+    if backend == "nccl":
+        torch.cuda.set_device(local)
+    dist.init_process_group(backend)
+    return dist.get_rank(), dist.get_world_size(), dist
+
+
+def barrier(dist):
+    if dist is not None:
+        dist.barrier()
+
+
+def max_over_ranks(x: float, dist) -> float:
+    if dist is None:
+        return x
+    import torch
+    dev = "cuda" if dist.get_backend() == "nccl" else "cpu"
+    t = torch.tensor([x], dtype=torch.float64, device=dev)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+# --- clocks -------------------------------------------------------------------------------
+
+class ClockSampler:
+    """nvidia-smi sampling of SM clocks and throttle reasons during the timed region."""
+    Q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+         "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+         "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, device_index: int):
+        self.device_index = device_index
+        self.proc = None
+
+    def __enter__(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--id={self.device_index}", f"--query-gpu={self.Q}",
+                 "--format=csv,noheader,nounits", "-lms", "200"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except OSError:
+            self.proc = None
+        return self
+
+    def __exit__(self, *exc):
+        self.lines = []
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                out, _ = self.proc.communicate(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+                out, _ = self.proc.communicate()
+            self.lines = [l for l in out.splitlines() if l.strip()]
+
+    def summary(self):
+        sm, mx, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in getattr(self, "lines", []):
+            f = [x.strip() for x in line.split(",")]
+            if len(f) < 9:
+                continue
+            try:
+                sm.append(float(f[1]))
+                mx.append(float(f[2]))
+            except ValueError:
+                continue
+            for name, val in zip(names, f[5:9]):
+                if val.lower().startswith("active"):
+                    reasons.add(name)
+        if not sm:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unsampled"], "samples": 0}
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx),
+                "reasons": sorted(reasons), "samples": len(sm)}
+
+
+# --- the step -------------------------------------------------------------------------------
+
+def generation_inputs(wl, step: int, n: int):
+    """Seeds and rewards of one generation (rewards stand in for rollouts)."""
+    seeds = I.population_seeds(n, generation=step)
+    rewards = I.rewards(wl.rewards if wl.rewards != "quadratic" else "uniform", n, seed=step)
+    return seeds, rewards
+
+
+def run_step(es, plan, wl, step, n, sigma, stream, timers=None):
+    """One ES generation through the C ABI. Returns the number of kernels launched."""
+    seeds, rewards = generation_inputs(wl, step, n)
+    launches = 0
+    for i in range(n):
+        if timers is not None:
+            timers.start("axpy")
+        es.es_perturb(plan, int(seeds[i]), sigma, stream)
+        # (rollout of the perturbed model happens here; its reward is an input)
+        es.es_restore(plan, int(seeds[i]), sigma, stream)
+        if timers is not None:
+            timers.stop("axpy", 2)
+        launches += 2
+    rhat = es.es_normalize_rewards(rewards, 1e-8)
+    coeffs = es.es_update_coeffs(rhat, wl.alpha, sigma, es.ES_SCALE_PAPER)
+    if timers is not None:
+        timers.start("update")
+    es.es_update(plan, seeds, coeffs, stream)
+    if timers is not None:
+        timers.stop("update", 1)
+    if np.any(coeffs != 0):
+        launches += 1
+    return launches
+
+
+class KernelTimers:
+    """CUDA-event pairs around kernel launches on the launching stream."""
+
+    def __init__(self, torch, stream):
+        self.torch = torch
+        self.stream = stream
+        self.pairs = {}
+        self._open = {}
+
+    def start(self, name):
+        e = self.torch.cuda.Event(enable_timing=True)
+        e.record(self.stream)
+        self._open[name] = e
+
+    def stop(self, name, count):
+        e = self.torch.cuda.Event(enable_timing=True)
+        e.record(self.stream)
+        self.pairs.setdefault(name, []).append((self._open.pop(name), e, count))
+
+    def mean_ms(self, name):
+        tot, cnt = 0.0, 0
+        for a, b, c in self.pairs.get(name, []):
+            tot += a.elapsed_time(b)
+            cnt += c
+        return tot / cnt if cnt else None
+
+    def total_ms(self, name):
+        return sum(a.elapsed_time(b) for a, b, _ in self.pairs.get(name, []))
+
+
+def run_ours(args, rank, world, dist):
+    import torch
+    from paper_2608_17310_gb300 import build, esopt as es
+
+    build.build_library()
+    dev_index = torch.cuda.current_device()
+    torch.cuda.init()
+    wl = I.WORKLOADS[args.workload]
+    n = args.population or wl.population
+    specs = I.shapes_for(args.workload)
+    dtype = torch.bfloat16 if wl.dtype == "bf16" else torch.float32
+    esize = 2 if wl.dtype == "bf16" else 4
+    params = I.init_params_torch(specs, dtype, "cuda", seed=0)
+    plan = es.plan_from_tensors(params)
+    P = plan.numel
+    stream = torch.cuda.current_stream()
+    s_handle = stream.cuda_stream
+    sigma0, sigmaT = wl.sigma, SIGMA_FINAL.get(args.workload, wl.sigma)
+
+    def sigma_at(t):
+        return float(np.float32(es.es_sigma_cosine(sigma0, sigmaT, t, SCHEDULE_T)))
+
+    for w in range(args.warmup):
+        run_step(es, plan, wl, w, n, sigma_at(w), s_handle)
+    torch.cuda.synchronize()
+    barrier(dist)
+    torch.cuda.synchronize()
+
+    timers = KernelTimers(torch, stream)
+    launches = 0
+    ev0 = torch.cuda.Event(enable_timing=True)
+    ev1 = torch.cuda.Event(enable_timing=True)
+    with ClockSampler(dev_index) as clk:
+        ev0.record(stream)
+        for k in range(args.steps):
+            t = args.warmup + k
+            launches += run_step(es, plan, wl, t, n, sigma_at(t), s_handle, timers)
+        ev1.record(stream)
+        torch.cuda.synchronize()
+    barrier(dist)
+    torch.cuda.synchronize()
+    ms = ev0.elapsed_time(ev1)
+    ms_max = max_over_ranks(ms, dist)
+    per_step_ms = ms_max / args.steps
+    value = world * P * n * args.steps / (ms_max / 1e3)
+
+    axpy_ms = timers.mean_ms("axpy")
+    upd_ms = timers.mean_ms("update")
+    hbm_gbs, sm_max_mhz, peak_src = peaks()
+    axpy_bytes = 2 * esize * P
+    axpy_gbs = axpy_bytes / (axpy_ms / 1e3) / 1e9
+    axpy_share = timers.total_ms("axpy") / ms
+    upd_share = timers.total_ms("update") / ms
+
+    e2e = None
+    if not args.no_e2e:
+        e2e = run_e2e(args, torch, es, plan, params, wl, n, esize, sigma_at, s_handle, dist, world)
+
+    cpu = None
+    if not args.no_cpu_baseline and rank == 0 and world == 1:
+        cpu = cpu_baseline(args.workload, n, sigma_at(args.warmup))
+
+    out = {
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": per_step_ms,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+        "dtype": wl.dtype, "data": "synthetic",
+        "config": {"workload": args.workload, "params": P, "population": n,
+                   "segments": len(specs), "description": wl.description,
+                   "sigma": sigma_at(args.warmup), "alpha": wl.alpha,
+                   "l2": "inputs larger than L2 (%.1f GB of parameters)" % (P * esize / 1e9),
+                   "parallelism": "replicas" if world > 1 else "single GPU"},
+        "roofline": {"bound": "hbm", "achieved": axpy_gbs, "peak": hbm_gbs, "unit": "GB/s",
+                     "frac": axpy_gbs / hbm_gbs, "traffic": None,
+                     "kernel": "axpy_noise_kernel<Bf16Io> (es_perturb / es_restore)",
+                     "peak_source": f"{peak_src} MEASURED_PEAKS.json hbm_gbs"},
+        "kernels": {
+            "axpy_noise": {"mean_ms": axpy_ms, "share": axpy_share,
+                           "gbs": axpy_gbs, "gauss_per_s": P / (axpy_ms / 1e3)},
+            "update": {"mean_ms": upd_ms, "share": upd_share,
+                       "gauss_per_s": P * n / (upd_ms / 1e3) if upd_ms else None,
+                       "gbs": axpy_bytes / (upd_ms / 1e3) / 1e9 if upd_ms else None},
+        },
+        "gpu_launches": launches,
+        "clocks": clk.summary(),
+        "e2e": e2e,
+        "cpu_baseline": cpu,
+    }
+    plan.close()
+    if rank == 0:
+        print(json.dumps(out), flush=True)
+
+
+def run_e2e(args, torch, es, plan, params, wl, n, esize, sigma_at, s_handle, dist, world):
+    """Same step with the parameters in pinned host memory: H2D copy, step, D2H copy."""
+    host = [torch.empty(p.shape, dtype=p.dtype, pin_memory=True) for p in params]
+    for h, p in zip(host, params):
+        h.copy_(p)
+    stream = torch.cuda.current_stream()
+    bytes_per_copy = sum(p.numel() for p in params) * esize
+
+    def one(t):
+        for h, p in zip(host, params):
+            p.copy_(h, non_blocking=True)
+        launches = run_step(es, plan, wl, t, n, sigma_at(t), s_handle)
+        for h, p in zip(host, params):
+            h.copy_(p, non_blocking=True)
+        return launches
+
+    one(0)
+    torch.cuda.synchronize()
+    barrier(dist)
+    e0 = torch.cuda.Event(enable_timing=True)
+    e1 = torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for k in range(args.e2e_steps):
+        one(args.warmup + k)
+    e1.record(stream)
+    torch.cuda.synchronize()
+    ms = max_over_ranks(e0.elapsed_time(e1), dist)
+    P = sum(p.numel() for p in params)
+    del host
+    return {"value": world * P * n * args.e2e_steps / (ms / 1e3), "unit": UNIT,
+            "steps": args.e2e_steps, "ms_per_step": ms / args.e2e_steps,
+            "h2d_bytes_per_step": bytes_per_copy, "d2h_bytes_per_step": bytes_per_copy}
+
+
+# --- CPU oracle (cpu_baseline leg and the reference arm) ---------------------------------
+
+def oracle_sample_step(workload: str, n: int, sigma: float, sample: int, step: int):
+    """One ES generation of the oracle on the first `sample` parameters of the
+    workload's first weight tensor. Returns elapsed seconds."""
+    from oracle import oracle as O
+    wl = I.WORKLOADS[workload]
+    specs = I.shapes_for(workload)
+    g = np.arange(min(sample, specs[0].numel), dtype=np.uint64)
+    theta32 = I.normal_f32(g.size, 0, 0.02)
+    dt = "bf16" if wl.dtype == "bf16" else "f32"
+    if dt == "bf16":
+        import torch
+        theta = torch.from_numpy(theta32).to(torch.bfloat16).view(torch.int16).numpy().view(np.uint16)
+    else:
+        theta = theta32
+    seeds, rewards = generation_inputs(wl, step, n)
+    t0 = time.perf_counter()
+    for i in range(n):
+        theta = O.perturb(theta, g, int(seeds[i]), sigma, dt)
+        theta = O.restore(theta, g, int(seeds[i]), sigma, dt)
+    coeffs = O.update_coeffs(O.zscore(rewards), wl.alpha, sigma, 0)
+    theta = O.update(theta, g, seeds, coeffs, dt)
+    return time.perf_counter() - t0, g.size
+
+
+def cpu_baseline(workload, n, sigma, sample=CPU_SAMPLE):
+    secs, m = oracle_sample_step(workload, n, sigma, sample, 0)
+    return {"value": m * n / secs, "unit": UNIT, "cores": 1, "kind": "oracle",
+            "sample": f"one generation (N={n} perturb+restore, update) on the first {m} "
+                      f"parameters of the {workload} set, single-threaded plain-C oracle; "
+                      f"{secs:.1f} s"}
+
+
+def run_reference(args, rank, world, dist):
+    if rank != 0:
+        return
+    wl = I.WORKLOADS[args.workload]
+    n = args.population or wl.population
+    sigma = float(np.float32(wl.sigma))
+    sample = 1 << 17
+    for w in range(args.warmup):
+        oracle_sample_step(args.workload, n, sigma, sample, w)
+    tot, m = 0.0, 0
+    for k in range(args.steps):
+        secs, m = oracle_sample_step(args.workload, n, sigma, sample, args.warmup + k)
+        tot += secs
+    value = m * n * args.steps / tot
+    desc = (f"each step: one generation (N={n}) of the plain-C oracle on the first {m} "
+            f"parameters of the {args.workload} set, single-threaded")
+    out = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world,
+           "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * tot / args.steps,
+           "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+           "dtype": wl.dtype, "data": "synthetic", "impl": "reference",
+           "config": {"workload": args.workload, "population": n, "sample_params": m},
+           "cpu_baseline": {"value": value, "unit": UNIT, "cores": 1, "kind": "oracle",
+                            "sample": desc},
+           "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0,
+                   "d2h_bytes_per_step": 0},
+           "gpu_launches": 0}
+    print(json.dumps(out), flush=True)
+
+
+def main():
+    args = parse()
+    rank, world, dist = dist_setup(args)
+    try:
+        if args.impl == "reference":
+            run_reference(args, rank, world, dist)
+        else:
+            run_ours(args, rank, world, dist)
+    finally:
+        if dist is not None:
+            dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

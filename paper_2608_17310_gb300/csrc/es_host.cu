@@ -1,0 +1,360 @@
+// C-ABI host layer: plan creation and validation, argument checks, the
+// host-side generation control of the paper (population z-score, cosine sigma
+// schedule, update coefficients) and dispatch to the kernels.
+#include <cuda_runtime.h>
+
+#include <algorithm>
+#include <cmath>
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+#include <new>
+#include <vector>
+
+#include "../../include/esopt.h"
+#include "es_internal.h"
+#include "es_noise.cuh"
+
+struct es_plan {
+  int device;
+  es_dtype_t dtype;
+  int nseg;
+  uint64_t numel;
+  uint64_t total_tiles;
+  esopt::SegDesc* d_segs;
+};
+
+namespace {
+
+thread_local char g_last_error[512] = "";
+
+es_status_t fail(es_status_t st, const char* fmt, ...) {
+  va_list ap;
+  va_start(ap, fmt);
+  std::vsnprintf(g_last_error, sizeof g_last_error, fmt, ap);
+  va_end(ap);
+  return st;
+}
+
+es_status_t ok() {
+  g_last_error[0] = '\0';
+  return ES_OK;
+}
+
+es_status_t cuda_fail(cudaError_t err, const char* what) {
+  return fail(ES_ERR_CUDA, "%s: %s (%s)", what, cudaGetErrorName(err), cudaGetErrorString(err));
+}
+
+size_t dtype_size(es_dtype_t dt) { return dt == ES_BF16 ? 2u : 4u; }
+
+es_status_t check_plan_device(const es_plan* plan) {
+  int cur = -1;
+  cudaError_t err = cudaGetDevice(&cur);
+  if (err != cudaSuccess) return cuda_fail(err, "cudaGetDevice");
+  if (cur != plan->device)
+    return fail(ES_ERR_WRONG_DEVICE, "plan lives on device %d but device %d is current",
+                plan->device, cur);
+  return ES_OK;
+}
+
+esopt::PlanView view(const es_plan* plan) {
+  return esopt::PlanView{plan->d_segs, plan->total_tiles, plan->dtype};
+}
+
+es_status_t axpy(es_plan_t plan, uint64_t seed, float scale, void* stream, const char* what) {
+  if (plan == nullptr) return fail(ES_ERR_INVALID_ARG, "%s: plan is NULL", what);
+  if (!std::isfinite(scale)) return fail(ES_ERR_NONFINITE, "%s: sigma is not finite", what);
+  es_status_t st = check_plan_device(plan);
+  if (st != ES_OK) return st;
+  cudaError_t err = esopt::launch_axpy_noise(view(plan), seed, scale,
+                                             static_cast<cudaStream_t>(stream));
+  if (err != cudaSuccess) return cuda_fail(err, what);
+  return ok();
+}
+
+}  // namespace
+
+extern "C" {
+
+es_status_t es_plan_create(const es_segment_t* segs, int nseg, es_dtype_t dtype,
+                           es_plan_t* out) {
+  if (out == nullptr) return fail(ES_ERR_INVALID_ARG, "es_plan_create: out is NULL");
+  *out = nullptr;
+  if (segs == nullptr || nseg < 1)
+    return fail(ES_ERR_INVALID_ARG, "es_plan_create: need at least one segment");
+  if (dtype != ES_BF16 && dtype != ES_FP32)
+    return fail(ES_ERR_INVALID_ARG, "es_plan_create: unknown dtype %d", static_cast<int>(dtype));
+  const size_t esize = dtype_size(dtype);
+  uint64_t total = 0;
+  for (int k = 0; k < nseg; ++k) {
+    const es_segment_t& s = segs[k];
+    if (s.data == nullptr || s.numel == 0)
+      return fail(ES_ERR_INVALID_ARG, "segment %d: NULL data or zero numel", k);
+    if (reinterpret_cast<uintptr_t>(s.data) % 16 != 0)
+      return fail(ES_ERR_ALIGNMENT, "segment %d: data is not 16-byte aligned", k);
+    if (s.index_base % 8 != 0)
+      return fail(ES_ERR_ALIGNMENT, "segment %d: index_base is not a multiple of 8", k);
+    if (s.index_base > UINT64_MAX - s.numel)
+      return fail(ES_ERR_INVALID_ARG, "segment %d: index range passes 2^64", k);
+    if (s.numel > UINT64_MAX / esize ||
+        reinterpret_cast<uintptr_t>(s.data) > UINTPTR_MAX - s.numel * esize)
+      return fail(ES_ERR_INVALID_ARG, "segment %d: byte range overflows", k);
+    if (total > UINT64_MAX - s.numel)
+      return fail(ES_ERR_INVALID_ARG, "total element count overflows");
+    total += s.numel;
+  }
+  // No two segments may share memory or global indices: each element must have
+  // one owner and one noise stream.
+  std::vector<int> order(nseg);
+  for (int k = 0; k < nseg; ++k) order[k] = k;
+  std::sort(order.begin(), order.end(),
+            [&](int a, int b) { return segs[a].index_base < segs[b].index_base; });
+  for (int k = 0; k + 1 < nseg; ++k) {
+    const es_segment_t& a = segs[order[k]];
+    const es_segment_t& b = segs[order[k + 1]];
+    if (a.index_base + a.numel > b.index_base)
+      return fail(ES_ERR_OVERLAP, "segments %d and %d overlap in index space", order[k],
+                  order[k + 1]);
+  }
+  std::sort(order.begin(), order.end(), [&](int a, int b) {
+    return reinterpret_cast<uintptr_t>(segs[a].data) < reinterpret_cast<uintptr_t>(segs[b].data);
+  });
+  for (int k = 0; k + 1 < nseg; ++k) {
+    const es_segment_t& a = segs[order[k]];
+    const es_segment_t& b = segs[order[k + 1]];
+    if (reinterpret_cast<uintptr_t>(a.data) + a.numel * esize > reinterpret_cast<uintptr_t>(b.data))
+      return fail(ES_ERR_OVERLAP, "segments %d and %d overlap in memory", order[k], order[k + 1]);
+  }
+
+  const uint64_t tile = esopt::tile_elems(dtype);
+  std::vector<esopt::SegDesc> table(static_cast<size_t>(nseg) + 1);
+  uint64_t tiles = 0;
+  for (int k = 0; k < nseg; ++k) {
+    table[k] = esopt::SegDesc{segs[k].data, segs[k].numel, segs[k].index_base, tiles};
+    tiles += (segs[k].numel + tile - 1) / tile;
+  }
+  table[nseg] = esopt::SegDesc{nullptr, 0, 0, tiles};
+
+  es_plan* plan = new (std::nothrow) es_plan{};
+  if (plan == nullptr) return fail(ES_ERR_NO_MEMORY, "es_plan_create: host allocation failed");
+  cudaError_t err = cudaGetDevice(&plan->device);
+  if (err != cudaSuccess) {
+    delete plan;
+    return cuda_fail(err, "cudaGetDevice");
+  }
+  const size_t bytes = table.size() * sizeof(esopt::SegDesc);
+  err = cudaMalloc(reinterpret_cast<void**>(&plan->d_segs), bytes);
+  if (err != cudaSuccess) {
+    delete plan;
+    cudaGetLastError();
+    return fail(err == cudaErrorMemoryAllocation ? ES_ERR_NO_MEMORY : ES_ERR_CUDA,
+                "cudaMalloc(segment table): %s", cudaGetErrorString(err));
+  }
+  err = cudaMemcpy(plan->d_segs, table.data(), bytes, cudaMemcpyHostToDevice);
+  if (err != cudaSuccess) {
+    cudaFree(plan->d_segs);
+    delete plan;
+    return cuda_fail(err, "cudaMemcpy(segment table)");
+  }
+  plan->dtype = dtype;
+  plan->nseg = nseg;
+  plan->numel = total;
+  plan->total_tiles = tiles;
+  *out = plan;
+  return ok();
+}
+
+es_status_t es_plan_destroy(es_plan_t plan) {
+  if (plan == nullptr) return ok();
+  int prev = -1;
+  cudaGetDevice(&prev);
+  if (prev != plan->device) cudaSetDevice(plan->device);
+  cudaError_t err = cudaFree(plan->d_segs);
+  if (prev != plan->device && prev >= 0) cudaSetDevice(prev);
+  delete plan;
+  if (err != cudaSuccess) return cuda_fail(err, "cudaFree(segment table)");
+  return ok();
+}
+
+uint64_t es_plan_numel(es_plan_t plan) { return plan == nullptr ? 0 : plan->numel; }
+
+uint64_t es_assign_index_bases(es_segment_t* segs, int nseg) {
+  if (segs == nullptr || nseg < 1) return 0;
+  uint64_t base = 0, end = 0;
+  for (int k = 0; k < nseg; ++k) {
+    segs[k].index_base = base;
+    end = base + segs[k].numel;
+    base = (end + 7) & ~static_cast<uint64_t>(7);
+  }
+  return end;
+}
+
+es_status_t es_noise_fill(uint64_t seed, uint64_t index_base, uint64_t n, float* out,
+                          void* stream) {
+  if (n == 0) return ok();
+  if (out == nullptr) return fail(ES_ERR_INVALID_ARG, "es_noise_fill: out is NULL");
+  if (reinterpret_cast<uintptr_t>(out) % 4 != 0)
+    return fail(ES_ERR_ALIGNMENT, "es_noise_fill: out is not 4-byte aligned");
+  if (index_base > UINT64_MAX - n)
+    return fail(ES_ERR_INVALID_ARG, "es_noise_fill: index range passes 2^64");
+  cudaError_t err = esopt::launch_noise_fill(seed, index_base, n, out,
+                                             static_cast<cudaStream_t>(stream));
+  if (err != cudaSuccess) return cuda_fail(err, "es_noise_fill");
+  return ok();
+}
+
+es_status_t es_noise_bits(uint64_t seed, uint64_t block_base, uint64_t nblocks, uint32_t* out,
+                          void* stream) {
+  if (nblocks == 0) return ok();
+  if (out == nullptr) return fail(ES_ERR_INVALID_ARG, "es_noise_bits: out is NULL");
+  if (reinterpret_cast<uintptr_t>(out) % 16 != 0)
+    return fail(ES_ERR_ALIGNMENT, "es_noise_bits: out is not 16-byte aligned");
+  const uint64_t kMaxBlock = uint64_t{1} << 62;
+  if (block_base > kMaxBlock || nblocks > kMaxBlock - block_base)
+    return fail(ES_ERR_INVALID_ARG, "es_noise_bits: block range passes 2^62");
+  cudaError_t err = esopt::launch_noise_bits(seed, block_base, nblocks, out,
+                                             static_cast<cudaStream_t>(stream));
+  if (err != cudaSuccess) return cuda_fail(err, "es_noise_bits");
+  return ok();
+}
+
+es_status_t es_perturb(es_plan_t plan, uint64_t seed, float sigma, void* stream) {
+  return axpy(plan, seed, sigma, stream, "es_perturb");
+}
+
+es_status_t es_restore(es_plan_t plan, uint64_t seed, float sigma, void* stream) {
+  return axpy(plan, seed, -sigma, stream, "es_restore");
+}
+
+es_status_t es_update(es_plan_t plan, const uint64_t* seeds, const float* coeffs, int n,
+                      void* stream) {
+  if (plan == nullptr) return fail(ES_ERR_INVALID_ARG, "es_update: plan is NULL");
+  if (seeds == nullptr || coeffs == nullptr || n < 1)
+    return fail(ES_ERR_INVALID_ARG, "es_update: need n >= 1 seeds and coefficients");
+  if (n > ES_MAX_SEEDS)
+    return fail(ES_ERR_TOO_MANY_SEEDS, "es_update: n = %d > ES_MAX_SEEDS = %d", n, ES_MAX_SEEDS);
+  esopt::UpdateArgs args;
+  std::memset(&args, 0, sizeof args);
+  int m = 0;
+  for (int i = 0; i < n; ++i) {
+    if (!std::isfinite(coeffs[i]))
+      return fail(ES_ERR_NONFINITE, "es_update: coefficient %d is not finite", i);
+    if (coeffs[i] == 0.0f) continue;  // adds exactly zero to every accumulator
+    const esopt::PhiloxKey key = esopt::philox_key(seeds[i]);
+    args.key[m][0] = key.k0;
+    args.key[m][1] = key.k1;
+    args.coeff[m] = coeffs[i];
+    ++m;
+  }
+  if (m == 0) return ok();  // no update: theta stays bit-identical
+  args.n = m;
+  es_status_t st = check_plan_device(plan);
+  if (st != ES_OK) return st;
+  cudaError_t err = esopt::launch_update(view(plan), args, static_cast<cudaStream_t>(stream));
+  if (err != cudaSuccess) return cuda_fail(err, "es_update");
+  return ok();
+}
+
+es_status_t es_normalize_rewards(const double* rewards, int n, double eps_z, double* rhat) {
+  if (rewards == nullptr || rhat == nullptr || n < 1)
+    return fail(ES_ERR_INVALID_ARG, "es_normalize_rewards: need n >= 1 rewards");
+  if (!(eps_z >= 0.0) || !std::isfinite(eps_z))
+    return fail(ES_ERR_INVALID_ARG, "es_normalize_rewards: eps_z must be finite and >= 0");
+  // Invalid (non-finite) rewards take the smallest finite reward of the batch.
+  int n_finite = 0;
+  double lo = 0.0, hi = 0.0;
+  for (int i = 0; i < n; ++i) {
+    if (!std::isfinite(rewards[i])) continue;
+    if (n_finite == 0 || rewards[i] < lo) lo = rewards[i];
+    if (n_finite == 0 || rewards[i] > hi) hi = rewards[i];
+    ++n_finite;
+  }
+  if (n_finite == 0 || lo == hi) {  // all invalid or all equal: no update
+    for (int i = 0; i < n; ++i) rhat[i] = 0.0;
+    return ok();
+  }
+  std::vector<double> r(rewards, rewards + n);
+  for (double& v : r)
+    if (!std::isfinite(v)) v = lo;
+  double mu = 0.0;
+  for (double v : r) mu += v;
+  mu /= n;
+  double var = 0.0;
+  for (double v : r) var += (v - mu) * (v - mu);
+  var /= n;
+  const double denom = std::sqrt(var) + eps_z;
+  for (int i = 0; i < n; ++i) rhat[i] = (r[i] - mu) / denom;
+  return ok();
+}
+
+double es_sigma_cosine(double sigma0, double sigmaT, int t, int T) {
+  if (T <= 0) return sigma0;
+  t = std::min(std::max(t, 0), T);
+  return sigmaT + (sigma0 - sigmaT) * (1.0 + std::cos(M_PI * t / T)) / 2.0;
+}
+
+static es_status_t coeffs_common(int n, double alpha, double sigma, es_scale_t mode,
+                                 double* denom_scale, const char* what) {
+  if (n < 1) return fail(ES_ERR_INVALID_ARG, "%s: n must be >= 1", what);
+  if (mode != ES_SCALE_PAPER && mode != ES_SCALE_CANONICAL)
+    return fail(ES_ERR_INVALID_ARG, "%s: unknown scale mode %d", what, static_cast<int>(mode));
+  if (!std::isfinite(alpha) || !std::isfinite(sigma))
+    return fail(ES_ERR_NONFINITE, "%s: alpha and sigma must be finite", what);
+  if (mode == ES_SCALE_CANONICAL && !(sigma > 0.0))
+    return fail(ES_ERR_INVALID_ARG, "%s: canonical scale needs sigma > 0", what);
+  *denom_scale = mode == ES_SCALE_CANONICAL ? sigma : 1.0;
+  return ES_OK;
+}
+
+es_status_t es_update_coeffs(const double* rhat, int n, double alpha, double sigma,
+                             es_scale_t mode, float* coeffs) {
+  if (rhat == nullptr || coeffs == nullptr)
+    return fail(ES_ERR_INVALID_ARG, "es_update_coeffs: NULL array");
+  double s = 1.0;
+  es_status_t st = coeffs_common(n, alpha, sigma, mode, &s, "es_update_coeffs");
+  if (st != ES_OK) return st;
+  const double denom = static_cast<double>(n) * s;
+  for (int i = 0; i < n; ++i) {
+    const double c = alpha * rhat[i] / denom;
+    if (!std::isfinite(c) || !std::isfinite(static_cast<float>(c)))
+      return fail(ES_ERR_NONFINITE, "es_update_coeffs: coefficient %d is not finite", i);
+    coeffs[i] = static_cast<float>(c);
+  }
+  return ok();
+}
+
+es_status_t es_fold_antithetic(const double* rhat_pos, const double* rhat_neg, int npairs,
+                               double alpha, double sigma, es_scale_t mode, float* coeffs) {
+  if (rhat_pos == nullptr || rhat_neg == nullptr || coeffs == nullptr)
+    return fail(ES_ERR_INVALID_ARG, "es_fold_antithetic: NULL array");
+  double s = 1.0;
+  es_status_t st = coeffs_common(npairs, alpha, sigma, mode, &s, "es_fold_antithetic");
+  if (st != ES_OK) return st;
+  const double denom = 2.0 * static_cast<double>(npairs) * s;
+  for (int i = 0; i < npairs; ++i) {
+    const double c = alpha * (rhat_pos[i] - rhat_neg[i]) / denom;
+    if (!std::isfinite(c) || !std::isfinite(static_cast<float>(c)))
+      return fail(ES_ERR_NONFINITE, "es_fold_antithetic: coefficient %d is not finite", i);
+    coeffs[i] = static_cast<float>(c);
+  }
+  return ok();
+}
+
+const char* es_status_string(es_status_t status) {
+  switch (status) {
+    case ES_OK: return "ES_OK";
+    case ES_ERR_INVALID_ARG: return "ES_ERR_INVALID_ARG: invalid argument";
+    case ES_ERR_ALIGNMENT: return "ES_ERR_ALIGNMENT: misaligned pointer or index base";
+    case ES_ERR_OVERLAP: return "ES_ERR_OVERLAP: segments overlap";
+    case ES_ERR_NONFINITE: return "ES_ERR_NONFINITE: non-finite scalar";
+    case ES_ERR_TOO_MANY_SEEDS: return "ES_ERR_TOO_MANY_SEEDS: more seeds than ES_MAX_SEEDS";
+    case ES_ERR_CUDA: return "ES_ERR_CUDA: CUDA error";
+    case ES_ERR_NO_MEMORY: return "ES_ERR_NO_MEMORY: allocation failed";
+    case ES_ERR_WRONG_DEVICE: return "ES_ERR_WRONG_DEVICE: plan belongs to another device";
+  }
+  return "unknown es_status_t";
+}
+
+const char* es_last_error(void) { return g_last_error; }
+
+}  // extern "C"

@@ -1,0 +1,60 @@
+// Internal interface between the C-ABI host layer (es_host.cpp) and the CUDA
+// kernels (es_kernels.cu). Not part of the public ABI.
+#pragma once
+
+#include <cuda_runtime.h>
+
+#include <cstdint>
+
+#include "../../include/esopt.h"
+
+namespace esopt {
+
+// Threads per CTA of the streaming kernels.
+constexpr int kBlockThreads = 256;
+// 16-byte vectors per thread per tile.
+constexpr int kVecsPerThread = 4;
+// Elements per 16-byte vector, per dtype.
+constexpr int vec_elems(es_dtype_t dt) { return dt == ES_BF16 ? 8 : 4; }
+// Elements per tile: a tile is the unit one CTA processes at a time; tiles
+// never straddle segments.
+constexpr uint64_t tile_elems(es_dtype_t dt) {
+  return static_cast<uint64_t>(kBlockThreads) * kVecsPerThread * vec_elems(dt);
+}
+
+// Device-side segment descriptor. A plan's table has nseg + 1 entries; the
+// last is a sentinel whose tile_begin is the total number of tiles.
+struct SegDesc {
+  void* data;           // 16-byte aligned storage of the segment
+  uint64_t numel;       // elements in the segment
+  uint64_t index_base;  // global index of element 0 (multiple of 8)
+  uint64_t tile_begin;  // first tile of the segment in the plan's tile space
+};
+static_assert(sizeof(SegDesc) == 32, "SegDesc layout");
+
+// Seeds and coefficients of one fused update, passed by value as a kernel
+// parameter and staged in shared memory by each CTA.
+struct UpdateArgs {
+  int n;
+  int pad_;
+  uint32_t key[ES_MAX_SEEDS][2];
+  float coeff[ES_MAX_SEEDS];
+};
+
+struct PlanView {
+  const SegDesc* segs;  // device table (nseg + 1 entries)
+  uint64_t total_tiles;
+  es_dtype_t dtype;
+};
+
+// Kernel launchers (es_kernels.cu). Each returns the launch's cudaError_t.
+cudaError_t launch_axpy_noise(const PlanView& plan, uint64_t seed, float scale,
+                              cudaStream_t stream);
+cudaError_t launch_update(const PlanView& plan, const UpdateArgs& args,
+                          cudaStream_t stream);
+cudaError_t launch_noise_bits(uint64_t seed, uint64_t block_base, uint64_t nblocks,
+                              uint32_t* out, cudaStream_t stream);
+cudaError_t launch_noise_fill(uint64_t seed, uint64_t index_base, uint64_t n,
+                              float* out, cudaStream_t stream);
+
+}  // namespace esopt

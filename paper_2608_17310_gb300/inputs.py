@@ -1,0 +1,168 @@
+"""Seeded synthetic inputs for the ES step: parameter-set shapes, initial
+parameters, population seeds and rewards.
+
+This module holds no arithmetic of the method (no noise generator, no
+normalisation, no update): it only draws inputs with numpy / torch generators
+from fixed seeds, so that the CUDA path and the CPU oracle can be fed the same
+values. Rollout rewards are out of scope, so rewards are drawn here from the
+distributions of the workloads instead.
+
+Workloads (the paper's LLM checkpoints are stood in for by random weights of
+the same shapes):
+  toy        1,048,576 fp32 values ~ N(0, 0.02^2), population 8 (seeds 1..8),
+             sigma 1e-3, alpha 1e-2, rewards Uniform[0,1]
+  quadratic  65,536 fp32, f(theta) = -||theta - theta*||^2, theta* ~ N(0,1),
+             32 antithetic pairs, sigma 0.05 -> 0.005 cosine over T = 200,
+             alpha 0.01
+  qwen4b     Qwen3.5-4B-shaped bf16 set: 36 layers, hidden 2560, 32 query and
+             8 KV heads of dim 128, SwiGLU 9728, vocab 151,936, tied
+             embeddings (4,022,458,880 parameters, 326 tensors); N = 16,
+             sigma 1e-3, Bernoulli(0.3) rewards
+  qwen27b    "27B"-shaped bf16 set: 64 layers, hidden 5120, 40 query and 8 KV
+             heads of dim 128, SwiGLU 17408, vocab 151,936, untied embeddings
+             (22,695,777,280 parameters, 579 tensors); N = 30, sigma_0 5e-4,
+             Uniform[0,1] rewards
+Weights ~ N(0, 0.02^2), norm weights = 1.
+"""
+from __future__ import annotations
+
+from dataclasses import dataclass
+from typing import List
+
+import numpy as np
+
+
+@dataclass(frozen=True)
+class TensorSpec:
+    name: str
+    numel: int
+    kind: str  # "weight" or "norm"
+
+
+def qwen_shapes(layers: int, hidden: int, q_heads: int, kv_heads: int, head_dim: int,
+                mlp: int, vocab: int, tied: bool) -> List[TensorSpec]:
+    """Parameter tensors of a Qwen-style decoder, in checkpoint order."""
+    specs = [TensorSpec("embed_tokens", vocab * hidden, "weight")]
+    q, kv = q_heads * head_dim, kv_heads * head_dim
+    for l in range(layers):
+        p = f"layers.{l}."
+        specs += [
+            TensorSpec(p + "input_layernorm", hidden, "norm"),
+            TensorSpec(p + "q_proj", hidden * q, "weight"),
+            TensorSpec(p + "k_proj", hidden * kv, "weight"),
+            TensorSpec(p + "v_proj", hidden * kv, "weight"),
+            TensorSpec(p + "o_proj", q * hidden, "weight"),
+            TensorSpec(p + "post_attention_layernorm", hidden, "norm"),
+            TensorSpec(p + "gate_proj", hidden * mlp, "weight"),
+            TensorSpec(p + "up_proj", hidden * mlp, "weight"),
+            TensorSpec(p + "down_proj", mlp * hidden, "weight"),
+        ]
+    specs.append(TensorSpec("norm", hidden, "norm"))
+    if not tied:
+        specs.append(TensorSpec("lm_head", vocab * hidden, "weight"))
+    return specs
+
+
+def qwen4b_shapes() -> List[TensorSpec]:
+    return qwen_shapes(36, 2560, 32, 8, 128, 9728, 151_936, tied=True)
+
+
+def qwen27b_shapes() -> List[TensorSpec]:
+    return qwen_shapes(64, 5120, 40, 8, 128, 17_408, 151_936, tied=False)
+
+
+@dataclass(frozen=True)
+class Workload:
+    name: str
+    dtype: str            # "bf16" or "f32"
+    population: int       # N seeds per update
+    sigma: float
+    alpha: float
+    rewards: str          # reward distribution
+    description: str
+
+
+WORKLOADS = {
+    "toy": Workload("toy", "f32", 8, 1e-3, 1e-2, "uniform",
+                    "1,048,576 fp32 ~ N(0, 0.02^2), N=8, seeds 1..8"),
+    "quadratic": Workload("quadratic", "f32", 32, 0.05, 0.01, "quadratic",
+                          "65,536 fp32 quadratic, 32 antithetic pairs, T=200"),
+    "qwen4b": Workload("qwen4b", "bf16", 16, 1e-3, 5e-4, "bernoulli0.3",
+                       "Qwen3.5-4B-shaped bf16 (4,022,458,880 params, 326 tensors), N=16"),
+    "qwen27b": Workload("qwen27b", "bf16", 30, 5e-4, 2.5e-4, "uniform",
+                        "27B-shaped bf16 (22,695,777,280 params, 579 tensors), N=30"),
+}
+
+
+def shapes_for(name: str) -> List[TensorSpec]:
+    if name == "qwen4b":
+        return qwen4b_shapes()
+    if name == "qwen27b":
+        return qwen27b_shapes()
+    if name == "toy":
+        return [TensorSpec("theta", 1 << 20, "weight")]
+    if name == "quadratic":
+        return [TensorSpec("theta", 1 << 16, "weight")]
+    raise KeyError(name)
+
+
+# --- draws ------------------------------------------------------------------------
+
+def normal_f32(n: int, seed: int, std: float = 1.0) -> np.ndarray:
+    """n fp32 draws of N(0, std^2) from numpy's PCG64 generator."""
+    return (std * np.random.default_rng(seed).standard_normal(n)).astype(np.float32)
+
+
+def toy_theta() -> np.ndarray:
+    """Toy workload: 1,048,576 fp32 values ~ N(0, 0.02^2) from seed 0."""
+    return normal_f32(1 << 20, 0, 0.02)
+
+
+def quadratic_problem(d: int = 1 << 16):
+    """(theta_0, theta_star) of the quadratic workload."""
+    return normal_f32(d, 0, 0.02), normal_f32(d, 12345, 1.0)
+
+
+def rewards(kind: str, n: int, seed: int) -> np.ndarray:
+    rng = np.random.default_rng(seed)
+    if kind == "uniform":
+        return rng.uniform(0.0, 1.0, n)
+    if kind.startswith("bernoulli"):
+        p = float(kind[len("bernoulli"):] or 0.5)
+        return (rng.uniform(0.0, 1.0, n) < p).astype(np.float64)
+    if kind == "normal":
+        return rng.standard_normal(n)
+    raise KeyError(kind)
+
+
+def population_seeds(n: int, generation: int = 0, first: int = 1) -> np.ndarray:
+    """Seeds of one generation: first + generation * 1000 + (0..n-1)."""
+    start = first + generation * 1000
+    return np.arange(start, start + n, dtype=np.uint64)
+
+
+def init_params_torch(specs: List[TensorSpec], dtype, device, seed: int = 0, std: float = 0.02):
+    """One torch tensor per spec: weights ~ N(0, std^2) from a seeded torch
+    generator on `device`, norm weights = 1."""
+    import torch
+    gen = torch.Generator(device=device)
+    gen.manual_seed(seed)
+    out = []
+    for s in specs:
+        t = torch.empty(s.numel, dtype=dtype, device=device)
+        if s.kind == "norm":
+            t.fill_(1.0)
+        else:
+            t.normal_(0.0, std, generator=gen)
+        out.append(t)
+    return out
+
+
+def sample_offsets(numel: int, n_random: int, seed: int, edge: int = 64) -> np.ndarray:
+    """Sorted unique local offsets: the first and last `edge` elements of a
+    tensor plus `n_random` uniform ones (parity checks at full size)."""
+    rng = np.random.default_rng(seed)
+    parts = [np.arange(min(edge, numel)), np.arange(max(0, numel - edge), numel)]
+    if n_random:
+        parts.append(rng.integers(0, numel, size=n_random))
+    return np.unique(np.concatenate(parts)).astype(np.int64)

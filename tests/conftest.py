@@ -18,3 +18,17 @@ def oracle():
     from oracle import oracle as O
     O.lib()
     return O
+
+
+@pytest.fixture(scope="session")
+def es():
+    """The CUDA library through its C-ABI binding. On a GPU run a missing GPU or
+    library is a failure, never a skip or a fallback."""
+    import torch
+    if not torch.cuda.is_available():
+        pytest.fail("a CUDA device is required for the gpu tests")
+    from paper_2608_17310_gb300 import build, esopt
+    build.build_library()
+    esopt._load()
+    torch.cuda.init()
+    return esopt

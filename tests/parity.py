@@ -1,0 +1,54 @@
+"""Comparison helpers shared by the parity tests (tolerances of the contract):
+Philox words bit-exact; eps within 1e-5 * max(1, |eps|); fp32 parameters within
+1e-5 relative plus the noise tolerance carried through the step
+(1e-5 * sum_i |c_i| max(1, |eps_i|) for theta + sum_i c_i eps_i, which keeps
+elements where theta and c eps cancel comparable); bf16 parameters within one
+ulp."""
+import numpy as np
+
+EPS_TOL = 1e-5
+F32_REL = 1e-5
+
+
+def assert_eps_close(got, want, what=""):
+    got = np.asarray(got, dtype=np.float64)
+    want = np.asarray(want, dtype=np.float64)
+    err = np.abs(got - want)
+    bound = EPS_TOL * np.maximum(1.0, np.abs(want))
+    bad = np.nonzero(~(err <= bound))[0]
+    assert bad.size == 0, (f"{what}: {bad.size} of {want.size} noise values out of tolerance; "
+                           f"first at {bad[:5]}: got {got[bad[:5]]} want {want[bad[:5]]}")
+
+
+def noise_abs_tol(eps_rows, coeffs):
+    """1e-5 * sum_i |c_i| * max(1, |eps_i|): the eps tolerance carried through
+    theta + sum_i c_i eps_i (eps_rows[i] is the oracle's eps of seed i)."""
+    tol = 0.0
+    for e, c in zip(eps_rows, coeffs):
+        tol = tol + EPS_TOL * abs(float(c)) * np.maximum(1.0, np.abs(e))
+    return tol
+
+
+def assert_f32_close(got, want, what="", abs_tol=0.0):
+    got = np.asarray(got, dtype=np.float64)
+    want = np.asarray(want, dtype=np.float64)
+    err = np.abs(got - want)
+    bound = F32_REL * np.abs(want) + abs_tol
+    bad = np.nonzero(~(err <= bound))[0]
+    assert bad.size == 0, (f"{what}: {bad.size} of {want.size} fp32 values out of tolerance; "
+                           f"first at {bad[:5]}: got {got[bad[:5]]} want {want[bad[:5]]}")
+
+
+def bf16_order(bits):
+    """Map bf16 bit patterns to integers that step by one per representable value."""
+    b = np.asarray(bits, dtype=np.uint16).astype(np.int64)
+    mag = b & 0x7FFF
+    return np.where(b & 0x8000, -mag, mag)
+
+
+def assert_bf16_within_ulp(got_bits, want_bits, what="", ulps=1):
+    d = np.abs(bf16_order(got_bits) - bf16_order(want_bits))
+    bad = np.nonzero(d > ulps)[0]
+    assert bad.size == 0, (f"{what}: {bad.size} of {d.size} bf16 values more than {ulps} ulp "
+                           f"apart; first at {bad[:5]}: got {np.asarray(got_bits)[bad[:5]]} "
+                           f"want {np.asarray(want_bits)[bad[:5]]}")

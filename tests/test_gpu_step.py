@@ -1,0 +1,186 @@
+"""GPU parity of perturb / restore / fused update through the C ABI, element by
+element against the oracle, on multi-segment plans with ragged tails, gaps in
+the index space and 64-bit indices, in bf16 and fp32 storage."""
+import numpy as np
+import pytest
+import torch
+
+from parity import assert_bf16_within_ulp, assert_f32_close, noise_abs_tol
+
+pytestmark = pytest.mark.gpu
+
+RAGGED = [1, 7, 8, 9, 8191, 8192, 8193, 20000, 100003, 4096 * 3 + 5]
+
+
+def make_params(dtype, numels, seed=0):
+    rng = np.random.default_rng(seed)
+    tensors = []
+    for n in numels:
+        v = torch.from_numpy((0.02 * rng.standard_normal(n)).astype(np.float32))
+        tensors.append((v.to(torch.bfloat16) if dtype == "bf16" else v).cuda())
+    return tensors
+
+
+def host_values(t):
+    c = t.detach().cpu()
+    if c.dtype == torch.bfloat16:
+        return c.view(torch.int16).numpy().view(np.uint16).copy()
+    return c.numpy().copy()
+
+
+def indices(plan_segs):
+    return [np.arange(s.index_base, s.index_base + s.numel, dtype=np.uint64) for s in plan_segs]
+
+
+def compare(dtype, got, want, what, abs_tol=0.0):
+    if dtype == "bf16":
+        assert_bf16_within_ulp(got, want, what)
+    else:
+        assert_f32_close(got, want, what, abs_tol)
+
+
+def ulp32(x):
+    return np.spacing(np.abs(np.asarray(x, dtype=np.float32))).astype(np.float64)
+
+
+def build_plan(es, tensors, bases=None):
+    segs = es.segments_from_tensors(tensors, bases)
+    plan = es.plan_from_tensors(tensors, [s.index_base for s in segs])
+    return plan, segs
+
+
+def _sparse64(n):
+    bases = [2**35 + k * 2**21 for k in range(n)]
+    bases[8] = 2**34 - 40      # 100003 elements straddle g = 2^34 (block j = 2^32)
+    bases[-1] = 2**61
+    return bases
+
+
+BASE_LAYOUTS = {
+    "packed": None,
+    # gaps, indices past 2^32 blocks (g >= 2^34) and one segment straddling g = 2^34
+    "sparse64": lambda numels: _sparse64(len(numels)),
+}
+
+
+@pytest.mark.parametrize("dtype", ["bf16", "f32"])
+@pytest.mark.parametrize("layout", list(BASE_LAYOUTS))
+def test_perturb_then_restore_match_oracle(es, oracle, dtype, layout):
+    tensors = make_params(dtype, RAGGED, seed=1)
+    bases = BASE_LAYOUTS[layout](RAGGED) if BASE_LAYOUTS[layout] else None
+    plan, segs = build_plan(es, tensors, bases)
+    before = [host_values(t) for t in tensors]
+    g = indices(segs)
+    seed, sigma = 2**40 + 17, 1e-3
+    es.es_perturb(plan, seed, sigma)
+    torch.cuda.synchronize()
+    perturbed = [host_values(t) for t in tensors]
+    eps = [oracle.noise_at(seed, gk) for gk in g]
+    for k in range(len(tensors)):
+        want = oracle.perturb(before[k], g[k], seed, sigma, dtype)
+        compare(dtype, perturbed[k], want, f"perturb seg {k} ({layout})",
+                noise_abs_tol([eps[k]], [sigma]))
+    es.es_restore(plan, seed, sigma)
+    torch.cuda.synchronize()
+    for k in range(len(tensors)):
+        got = host_values(tensors[k])
+        want = oracle.restore(perturbed[k], g[k], seed, sigma, dtype)   # step by step
+        compare(dtype, got, want, f"restore seg {k} ({layout})", noise_abs_tol([eps[k]], [sigma]))
+        if dtype == "f32":     # the round trip returns theta within one rounding
+            bound = 2 * ulp32(np.maximum(np.abs(before[k]), sigma * np.abs(eps[k])))
+            assert np.all(np.abs(got.astype(np.float64) - before[k]) <= bound), f"round trip {k}"
+    plan.close()
+
+
+@pytest.mark.parametrize("dtype", ["bf16", "f32"])
+@pytest.mark.parametrize("nseeds", [1, 2, 3, 8, 30, 129, 256])
+def test_update_matches_oracle(es, oracle, dtype, nseeds):
+    numels = [9, 8193, 20000, 4096 * 3 + 5]
+    tensors = make_params(dtype, numels, seed=2)
+    plan, segs = build_plan(es, tensors, [8, 2**34 - 1024, 2**36, 2**50])
+    before = [host_values(t) for t in tensors]
+    rng = np.random.default_rng(nseeds)
+    seeds = rng.integers(0, 2**63, size=nseeds, dtype=np.uint64)
+    coeffs = (1e-3 * rng.standard_normal(nseeds)).astype(np.float32)
+    if nseeds > 2:
+        coeffs[1] = 0.0          # a zero coefficient is skipped without changing the result
+    es.es_update(plan, seeds, coeffs)
+    torch.cuda.synchronize()
+    g = indices(segs)
+    for k in range(len(tensors)):
+        want = oracle.update(before[k], g[k], seeds, coeffs, dtype)
+        tol = noise_abs_tol([oracle.noise_at(int(s), g[k]) for s in seeds], coeffs) \
+            if dtype == "f32" else 0.0
+        compare(dtype, host_values(tensors[k]), want, f"update N={nseeds} seg {k}", tol)
+    plan.close()
+
+
+@pytest.mark.parametrize("dtype", ["bf16", "f32"])
+def test_update_is_deterministic_and_launch_independent(es, dtype):
+    tensors = make_params(dtype, [100003, 77], seed=3)
+    copies = [t.clone() for t in tensors]
+    plan_a, _ = build_plan(es, tensors)
+    plan_b, _ = build_plan(es, copies)
+    seeds, coeffs = np.arange(1, 17, dtype=np.uint64), np.linspace(-1e-3, 1e-3, 16, dtype=np.float32)
+    es.es_update(plan_a, seeds, coeffs)
+    s = torch.cuda.Stream()
+    with torch.cuda.stream(s):
+        es.es_update(plan_b, seeds, coeffs, stream=s)
+    torch.cuda.synchronize()
+    for a, b in zip(tensors, copies):
+        assert torch.equal(a.view(torch.int16 if dtype == "bf16" else torch.int32),
+                           b.view(torch.int16 if dtype == "bf16" else torch.int32))
+
+
+def test_all_zero_coefficients_leave_theta_bit_identical(es):
+    tensors = make_params("bf16", [8192, 5], seed=4)
+    ref = [t.clone() for t in tensors]
+    plan, _ = build_plan(es, tensors)
+    es.es_update(plan, np.arange(8, dtype=np.uint64), np.zeros(8, np.float32))
+    torch.cuda.synchronize()
+    assert all(torch.equal(a.view(torch.int16), b.view(torch.int16)) for a, b in zip(tensors, ref))
+
+
+def test_step_argument_errors(es):
+    t = make_params("bf16", [64], seed=5)[0]
+    plan, _ = build_plan(es, [t])
+    with pytest.raises(es.EsError) as ei:
+        es.es_perturb(plan, 1, float("nan"))
+    assert ei.value.status == es.ES_ERR_NONFINITE
+    with pytest.raises(es.EsError) as ei:
+        es.es_restore(plan, 1, float("inf"))
+    assert ei.value.status == es.ES_ERR_NONFINITE
+    with pytest.raises(es.EsError) as ei:
+        es.es_update(plan, np.arange(257, dtype=np.uint64), np.ones(257, np.float32))
+    assert ei.value.status == es.ES_ERR_TOO_MANY_SEEDS
+    with pytest.raises(es.EsError) as ei:
+        es.es_update(plan, [1, 2], np.array([1.0, np.nan], np.float32))
+    assert ei.value.status == es.ES_ERR_NONFINITE
+    with pytest.raises(es.EsError) as ei:
+        es.es_update(plan, [], [])
+    assert ei.value.status == es.ES_ERR_INVALID_ARG
+    # misaligned segment: data pointer one bf16 element into the tensor
+    with pytest.raises(es.EsError) as ei:
+        es.es_plan_create([es.Segment(t.data_ptr() + 2, 8, 0)], es.ES_BF16)
+    assert ei.value.status == es.ES_ERR_ALIGNMENT
+    # two segments sharing memory
+    with pytest.raises(es.EsError) as ei:
+        es.es_plan_create([es.Segment(t.data_ptr(), 32, 0), es.Segment(t.data_ptr() + 32, 32, 64)],
+                          es.ES_BF16)
+    assert ei.value.status == es.ES_ERR_OVERLAP
+    plan.close()
+
+
+def test_max_population_update(es, oracle):
+    t = make_params("f32", [4099], seed=6)[0]
+    plan, segs = build_plan(es, [t])
+    before = host_values(t)
+    seeds = np.arange(10**6, 10**6 + es.ES_MAX_SEEDS, dtype=np.uint64)
+    coeffs = np.full(es.ES_MAX_SEEDS, 1e-4, np.float32)
+    es.es_update(plan, seeds, coeffs)
+    torch.cuda.synchronize()
+    g = indices(segs)[0]
+    want = oracle.update(before, g, seeds, coeffs, "f32")
+    tol = noise_abs_tol([oracle.noise_at(int(s), g) for s in seeds], coeffs)
+    assert_f32_close(host_values(t), want, "N=256", tol)
+    plan.close()
