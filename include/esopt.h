@@ -232,6 +232,40 @@ es_status_t es_fold_antithetic(const double* rhat_pos, const double* rhat_neg,
                                int npairs, double alpha, double sigma,
                                es_scale_t mode, float* coeffs);
 
+/*
+ * Perturb without allocating. The paper has no counterpart to this entry
+ * point; it exists for callers that must not allocate device memory after
+ * start-up: a process whose device memory is handed out by its own pool or
+ * caching allocator (a stray cudaMalloc there fragments memory the pool
+ * counts as free, and cudaMalloc/cudaFree can synchronise the device), or a
+ * latency-bound loop that may not call into the allocator at all.
+ *
+ * theta[g] <- round(theta[g] + sigma * eps_seed[g]) over the given segments,
+ * exactly as es_perturb on a plan made from the same segments; pass -sigma to
+ * restore. Segments follow the rules of es_plan_create (16-byte aligned data,
+ * index bases multiples of 8, no overlap) and are validated on every call.
+ *
+ * Instead of a plan's table, the segment table is copied (cudaMemcpyAsync on
+ * `stream`) into one static device array of ES_STATIC_MAX_SEGMENTS + 1
+ * descriptors (about 32 KB), which every device that loads the library holds
+ * until the process exits. The entry point calls no cudaMalloc, cudaFree or
+ * other allocating routine, and uses about 36 KB of host stack.
+ *   - More than ES_STATIC_MAX_SEGMENTS segments: ES_ERR_INVALID_ARG, nothing
+ *     is launched.
+ *   - All calls share the one array and each call rewrites it whole (nothing
+ *     in it needs to start at zero); it keeps the last call's table. Calls
+ *     that overlap on the GPU (on different streams, or from several host
+ *     threads without ordering) race on that array and must not be issued.
+ *   - The first call on each device looks up the array's device address
+ *     (cudaGetSymbolAddress) with that device current; make that first call
+ *     before any stream capture.
+ * Errors: ES_ERR_INVALID_ARG, ES_ERR_ALIGNMENT, ES_ERR_OVERLAP,
+ * ES_ERR_NONFINITE, ES_ERR_CUDA.
+ */
+#define ES_STATIC_MAX_SEGMENTS 1024
+es_status_t es_perturb_noalloc(const es_segment_t* segs, int nseg, es_dtype_t dtype,
+                               uint64_t seed, float sigma, void* stream);
+
 /* Static description of a status code. */
 const char* es_status_string(es_status_t status);
 

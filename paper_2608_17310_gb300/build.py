@@ -21,7 +21,7 @@ INCLUDE = os.path.join(ROOT, "include")
 BUILD = os.path.join(PKG, "_build")
 LIB = os.path.join(BUILD, "libesopt.so")
 
-SOURCES = ["es_host.cu", "es_kernels.cu"]
+SOURCES = ["es_host.cu", "es_kernels.cu", "es_noalloc.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 NVCC_FLAGS = ["-std=c++17", "-O3", "-lineinfo", "-Xcompiler", "-fPIC,-O2",
               "-Xptxas", "-v", f"-I{INCLUDE}"]

@@ -74,6 +74,15 @@ es_status_t axpy(es_plan_t plan, uint64_t seed, float scale, void* stream, const
 
 }  // namespace
 
+namespace esopt {
+// Records `message` as the calling thread's es_last_error() text and returns
+// `status` (ES_OK clears the text). For entry points defined in other files.
+es_status_t record_status(es_status_t status, const char* message) {
+  if (status == ES_OK) return ok();
+  return fail(status, "%s", message);
+}
+}  // namespace esopt
+
 extern "C" {
 
 es_status_t es_plan_create(const es_segment_t* segs, int nseg, es_dtype_t dtype,

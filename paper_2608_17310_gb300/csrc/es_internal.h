@@ -57,4 +57,7 @@ cudaError_t launch_noise_bits(uint64_t seed, uint64_t block_base, uint64_t nbloc
 cudaError_t launch_noise_fill(uint64_t seed, uint64_t index_base, uint64_t n,
                               float* out, cudaStream_t stream);
 
+// Sets the calling thread's es_last_error() text (es_host.cu).
+es_status_t record_status(es_status_t status, const char* message);
+
 }  // namespace esopt

@@ -25,6 +25,7 @@ _PKG = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.path.join(_PKG, "_build", "libesopt.so")
 
 ES_MAX_SEEDS = 256
+ES_STATIC_MAX_SEGMENTS = 1024
 
 ES_OK = 0
 ES_ERR_INVALID_ARG = 1
@@ -83,6 +84,7 @@ def _load() -> ctypes.CDLL:
         "es_sigma_cosine": (f64, [f64, f64, i32, i32]),
         "es_update_coeffs": (i32, [P(f64), i32, f64, f64, i32, P(f32)]),
         "es_fold_antithetic": (i32, [P(f64), P(f64), i32, f64, f64, i32, P(f32)]),
+        "es_perturb_noalloc": (i32, [P(es_segment_t), i32, i32, u64, f32, vp]),
         "es_status_string": (ctypes.c_char_p, [i32]),
         "es_last_error": (ctypes.c_char_p, []),
     }
@@ -256,6 +258,15 @@ def es_update(plan: Plan, seeds, coeffs, stream=None) -> None:
     _check(_load().es_update(plan.handle, s.ctypes.data_as(ctypes.POINTER(ctypes.c_uint64)),
                              c.ctypes.data_as(ctypes.POINTER(ctypes.c_float)), s.size,
                              _stream(stream)), "es_update")
+
+
+def es_perturb_noalloc(segments: Sequence[Segment], dtype: int, seed: int, sigma: float,
+                       stream=None) -> None:
+    """Perturb (or, with -sigma, restore) without a plan and without any device
+    allocation; the segment table goes to the library's static device array."""
+    arr = _seg_array(segments)
+    _check(_load().es_perturb_noalloc(arr, len(segments), dtype, seed, sigma, _stream(stream)),
+           "es_perturb_noalloc")
 
 
 # --- host-side generation control ---------------------------------------------------

@@ -1,0 +1,65 @@
+"""es_perturb_noalloc: the perturb/restore pass for callers that cannot
+allocate device memory (a process whose device memory belongs to its own pool
+allocator, or a loop that must not call into the allocator). It must give the
+same parameters as the plan-based es_perturb / es_restore, call after call.
+
+Kept in a file that is collected last, so a run that stops at the first
+failure has run every other test before this one.
+"""
+import numpy as np
+import pytest
+import torch
+
+from parity import assert_bf16_within_ulp, assert_f32_close, noise_abs_tol
+
+pytestmark = pytest.mark.gpu
+
+NUMELS = [7, 2560, 8193, 20000, 100003]
+
+
+def _params(dtype, seed):
+    rng = np.random.default_rng(seed)
+    out = []
+    for n in NUMELS:
+        v = torch.from_numpy((0.02 * rng.standard_normal(n)).astype(np.float32))
+        out.append((v.to(torch.bfloat16) if dtype == "bf16" else v).cuda())
+    return out
+
+
+def _host(t):
+    c = t.cpu()
+    return c.view(torch.int16).numpy().view(np.uint16) if c.dtype == torch.bfloat16 else c.numpy()
+
+
+@pytest.mark.parametrize("dtype", ["bf16", "f32"])
+def test_noalloc_matches_plan_entry_points_on_two_calls_in_a_row(es, oracle, dtype):
+    a = _params(dtype, 11)
+    b = [t.clone() for t in a]
+    plan = es.plan_from_tensors(a)
+    bases = [s.index_base for s in es.segments_from_tensors(a)]
+    segs_b = es.segments_from_tensors(b, bases)
+    code = es.ES_BF16 if dtype == "bf16" else es.ES_FP32
+    seed, sigma = 2**33 + 5, 1e-3
+    # call 1: perturb; call 2: restore (-sigma) of the same seed
+    for k, (plan_call, scale) in enumerate([(es.es_perturb, sigma), (es.es_restore, -sigma)]):
+        plan_call(plan, seed, sigma)
+        es.es_perturb_noalloc(segs_b, code, seed, scale)
+        torch.cuda.synchronize()
+        for j, (x, y) in enumerate(zip(a, b)):
+            if dtype == "bf16":
+                assert_bf16_within_ulp(_host(y), _host(x), f"call {k + 1} segment {j}")
+            else:
+                g = np.arange(bases[j], bases[j] + x.numel(), dtype=np.uint64)
+                tol = noise_abs_tol([oracle.noise_at(seed, g)], [sigma])
+                assert_f32_close(_host(y), _host(x), f"call {k + 1} segment {j}", tol)
+    plan.close()
+
+
+def test_noalloc_rejects_more_segments_than_its_static_table(es):
+    # Rejected before any device work: the pointers are never dereferenced.
+    n = es.ES_STATIC_MAX_SEGMENTS + 1
+    segs = [es.Segment(0x100000 + 16 * k, 1, 8 * k) for k in range(n)]
+    with pytest.raises(es.EsError) as ei:
+        es.es_perturb_noalloc(segs, es.ES_BF16, 1, 1e-3)
+    assert ei.value.status == es.ES_ERR_INVALID_ARG
+    assert "ES_STATIC_MAX_SEGMENTS" in str(ei.value)
