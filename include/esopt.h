@@ -153,6 +153,19 @@ es_status_t es_noise_bits(uint64_t seed, uint64_t block_base, uint64_t nblocks,
                           uint32_t* out, void* stream);
 
 /*
+ * The uniform mapping and Box-Muller transform of the generator applied to
+ * caller-supplied word pairs, in fp32, exactly as every device entry point
+ * applies them to Philox words:
+ *   out[2k]   = r cos(2 pi u(words[2k+1])),  out[2k+1] = r sin(2 pi u(words[2k+1])),
+ *   r = sqrt(-2 ln u(words[2k])),  u(x) = (2 (x >> 9) + 1) / 2^24.
+ * Each word matters only through its top 23 bits, so this lets the transform
+ * be checked over its whole input domain. `words` and `out` are device
+ * buffers of 2 * npairs entries, 8-byte aligned; npairs = 0 is a no-op.
+ * Errors: ES_ERR_INVALID_ARG, ES_ERR_ALIGNMENT, ES_ERR_CUDA.
+ */
+es_status_t es_box_muller(const uint32_t* words, uint64_t npairs, float* out, void* stream);
+
+/*
  * Perturb in place (§3; App. D.6 "applies theta + sigma_t eps_i"):
  * theta[g] <- round(theta[g] + sigma * eps_seed[g]) for every element of every
  * segment, with the product and sum in fp32 (one fused multiply-add) and one

@@ -109,16 +109,29 @@ double oracle_uniform(uint32_t x) {
  * Output words (x0, x1) of a block form the first pair (elements 4j, 4j+1),
  * (x2, x3) the second (elements 4j+2, 4j+3).
  */
+void oracle_box_muller(uint32_t x_a, uint32_t x_b, double out[2]) {
+  double u_a = oracle_uniform(x_a);
+  double u_b = oracle_uniform(x_b);
+  double r = sqrt(-2.0 * log(u_a));
+  double phi = 2.0 * M_PI * u_b;
+  out[0] = r * cos(phi);
+  out[1] = r * sin(phi);
+}
+
+/* Box-Muller on word pairs: out[2k], out[2k+1] from (words[2k], words[2k+1]). */
+void oracle_box_muller_fill(const uint32_t* words, uint64_t npairs, double* out) {
+  for (uint64_t k = 0; k < npairs; ++k)
+    oracle_box_muller(words[2 * k], words[2 * k + 1], out + 2 * k);
+}
+
 double oracle_gaussian(uint64_t seed, uint64_t g) {
   uint32_t x[4];
   oracle_noise_block(seed, g >> 2, x);
   int k = (int)(g & 3u);
   int pair = k >> 1;
-  double u_a = oracle_uniform(x[2 * pair]);
-  double u_b = oracle_uniform(x[2 * pair + 1]);
-  double r = sqrt(-2.0 * log(u_a));
-  double phi = 2.0 * M_PI * u_b;
-  return (k & 1) ? r * sin(phi) : r * cos(phi);
+  double e[2];
+  oracle_box_muller(x[2 * pair], x[2 * pair + 1], e);
+  return e[k & 1];
 }
 
 /* eps_seed[g] for g in [index_base, index_base + n). */

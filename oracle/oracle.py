@@ -53,6 +53,7 @@ def lib() -> ctypes.CDLL:
             L.oracle_noise_block.argtypes = [ctypes.c_uint64, ctypes.c_uint64, _u32p]
             L.oracle_uniform.argtypes = [ctypes.c_uint32]
             L.oracle_uniform.restype = ctypes.c_double
+            L.oracle_box_muller_fill.argtypes = [_u32p, ctypes.c_uint64, _f64p]
             L.oracle_gaussian.argtypes = [ctypes.c_uint64, ctypes.c_uint64]
             L.oracle_gaussian.restype = ctypes.c_double
             L.oracle_noise_fill.argtypes = [ctypes.c_uint64, ctypes.c_uint64,
@@ -114,6 +115,15 @@ def noise_block(seed: int, j: int) -> np.ndarray:
 
 def uniform(x: int) -> float:
     return lib().oracle_uniform(x)
+
+
+def box_muller(words: np.ndarray) -> np.ndarray:
+    """Box-Muller of word pairs (words[2k] -> radius, words[2k+1] -> angle)."""
+    w = np.ascontiguousarray(words, dtype=np.uint32)
+    out = np.empty(w.size, dtype=np.float64)
+    if w.size:
+        lib().oracle_box_muller_fill(_ptr(w, _u32p), w.size // 2, _ptr(out, _f64p))
+    return out
 
 
 def gaussian(seed: int, g: int) -> float:

@@ -227,6 +227,19 @@ es_status_t es_noise_bits(uint64_t seed, uint64_t block_base, uint64_t nblocks, 
   return ok();
 }
 
+es_status_t es_box_muller(const uint32_t* words, uint64_t npairs, float* out, void* stream) {
+  if (npairs == 0) return ok();
+  if (words == nullptr || out == nullptr)
+    return fail(ES_ERR_INVALID_ARG, "es_box_muller: NULL buffer");
+  if (reinterpret_cast<uintptr_t>(words) % 8 != 0 || reinterpret_cast<uintptr_t>(out) % 8 != 0)
+    return fail(ES_ERR_ALIGNMENT, "es_box_muller: buffers must be 8-byte aligned");
+  if (npairs > (UINT64_MAX >> 4))
+    return fail(ES_ERR_INVALID_ARG, "es_box_muller: npairs too large");
+  cudaError_t err = esopt::launch_box_muller(words, npairs, out, static_cast<cudaStream_t>(stream));
+  if (err != cudaSuccess) return cuda_fail(err, "es_box_muller");
+  return ok();
+}
+
 es_status_t es_perturb(es_plan_t plan, uint64_t seed, float sigma, void* stream) {
   return axpy(plan, seed, sigma, stream, "es_perturb");
 }

@@ -54,6 +54,8 @@ cudaError_t launch_update(const PlanView& plan, const UpdateArgs& args,
                           cudaStream_t stream);
 cudaError_t launch_noise_bits(uint64_t seed, uint64_t block_base, uint64_t nblocks,
                               uint32_t* out, cudaStream_t stream);
+cudaError_t launch_box_muller(const uint32_t* words, uint64_t npairs, float* out,
+                              cudaStream_t stream);
 cudaError_t launch_noise_fill(uint64_t seed, uint64_t index_base, uint64_t n,
                               float* out, cudaStream_t stream);
 

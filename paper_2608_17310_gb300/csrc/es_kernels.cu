@@ -220,6 +220,17 @@ noise_bits_kernel(uint64_t block_base, uint64_t nblocks, PhiloxKey key, uint4* _
     out[t] = philox_block(block_base + t, key);
 }
 
+// out[2k], out[2k+1] = Box-Muller pair of words[2k], words[2k+1].
+__global__ void __launch_bounds__(kBlockThreads)
+box_muller_kernel(const uint2* __restrict__ words, uint64_t npairs, float2* __restrict__ out) {
+  const uint64_t stride = static_cast<uint64_t>(gridDim.x) * blockDim.x;
+  for (uint64_t k = static_cast<uint64_t>(blockIdx.x) * blockDim.x + threadIdx.x; k < npairs;
+       k += stride) {
+    const uint2 w = words[k];
+    out[k] = box_muller(w.x, w.y);
+  }
+}
+
 // Persistent grid: every SM filled to the kernel's occupancy, never more
 // CTAs than tiles.
 template <class K>
@@ -271,6 +282,15 @@ cudaError_t launch_noise_bits(uint64_t seed, uint64_t block_base, uint64_t nbloc
   const int grid = persistent_grid(noise_bits_kernel, ctas);
   noise_bits_kernel<<<grid, kBlockThreads, 0, stream>>>(block_base, nblocks, philox_key(seed),
                                                         reinterpret_cast<uint4*>(out));
+  return cudaGetLastError();
+}
+
+cudaError_t launch_box_muller(const uint32_t* words, uint64_t npairs, float* out,
+                              cudaStream_t stream) {
+  const uint64_t ctas = (npairs + kBlockThreads - 1) / kBlockThreads;
+  const int grid = persistent_grid(box_muller_kernel, ctas);
+  box_muller_kernel<<<grid, kBlockThreads, 0, stream>>>(reinterpret_cast<const uint2*>(words),
+                                                        npairs, reinterpret_cast<float2*>(out));
   return cudaGetLastError();
 }
 

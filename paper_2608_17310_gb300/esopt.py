@@ -77,6 +77,7 @@ def _load() -> ctypes.CDLL:
         "es_assign_index_bases": (u64, [P(es_segment_t), i32]),
         "es_noise_fill": (i32, [u64, u64, u64, vp, vp]),
         "es_noise_bits": (i32, [u64, u64, u64, vp, vp]),
+        "es_box_muller": (i32, [vp, u64, vp, vp]),
         "es_perturb": (i32, [vp, u64, f32, vp]),
         "es_restore": (i32, [vp, u64, f32, vp]),
         "es_update": (i32, [vp, P(u64), P(f32), i32, vp]),
@@ -240,6 +241,11 @@ def es_noise_fill(seed: int, index_base: int, n: int, out, stream=None) -> None:
 def es_noise_bits(seed: int, block_base: int, nblocks: int, out, stream=None) -> None:
     _check(_load().es_noise_bits(seed, block_base, nblocks, _ptr(out), _stream(stream)),
            "es_noise_bits")
+
+
+def es_box_muller(words, npairs: int, out, stream=None) -> None:
+    _check(_load().es_box_muller(_ptr(words), npairs, _ptr(out), _stream(stream)),
+           "es_box_muller")
 
 
 def es_perturb(plan: Plan, seed: int, sigma: float, stream=None) -> None:

@@ -91,6 +91,9 @@ WORKLOADS = {
                        "Qwen3.5-4B-shaped bf16 (4,022,458,880 params, 326 tensors), N=16"),
     "qwen27b": Workload("qwen27b", "bf16", 30, 5e-4, 2.5e-4, "uniform",
                         "27B-shaped bf16 (22,695,777,280 params, 579 tensors), N=30"),
+    # profiling case: the 4B shapes cut to 4 layers (about 1.6 GB, larger than L2)
+    "qwen4b_4layer": Workload("qwen4b_4layer", "bf16", 16, 1e-3, 5e-4, "bernoulli0.3",
+                              "Qwen3.5-4B shapes, 4 layers (792,680,960 params, 38 tensors), N=16"),
 }
 
 
@@ -99,6 +102,8 @@ def shapes_for(name: str) -> List[TensorSpec]:
         return qwen4b_shapes()
     if name == "qwen27b":
         return qwen27b_shapes()
+    if name == "qwen4b_4layer":
+        return qwen_shapes(4, 2560, 32, 8, 128, 9728, 151_936, tied=True)
     if name == "toy":
         return [TensorSpec("theta", 1 << 20, "weight")]
     if name == "quadratic":

@@ -34,7 +34,7 @@ def indices(plan_segs):
 
 def compare(dtype, got, want, what, abs_tol=0.0):
     if dtype == "bf16":
-        assert_bf16_within_ulp(got, want, what)
+        assert_bf16_within_ulp(got, want, what, abs_tol=abs_tol)
     else:
         assert_f32_close(got, want, what, abs_tol)
 
@@ -109,8 +109,7 @@ def test_update_matches_oracle(es, oracle, dtype, nseeds):
     g = indices(segs)
     for k in range(len(tensors)):
         want = oracle.update(before[k], g[k], seeds, coeffs, dtype)
-        tol = noise_abs_tol([oracle.noise_at(int(s), g[k]) for s in seeds], coeffs) \
-            if dtype == "f32" else 0.0
+        tol = noise_abs_tol([oracle.noise_at(int(s), g[k]) for s in seeds], coeffs)
         compare(dtype, host_values(tensors[k]), want, f"update N={nseeds} seg {k}", tol)
     plan.close()
 
