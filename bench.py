@@ -49,6 +49,8 @@ def parse():
     p.add_argument("--no-e2e", action="store_true")
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--e2e-steps", type=int, default=2)
+    p.add_argument("--unfused", action="store_true",
+                   help="separate es_restore / es_perturb launches instead of es_restore_perturb")
     return p.parse_args()
 
 
@@ -155,29 +157,38 @@ def generation_inputs(wl, step: int, n: int):
     return seeds, rewards
 
 
-def run_step(es, plan, wl, step, n, sigma, stream, timers=None):
+def run_step(es, plan, wl, step, n, sigma, stream, timers=None, fused=True):
     """One ES generation through the C ABI. Returns the number of kernels launched."""
     seeds, rewards = generation_inputs(wl, step, n)
-    launches = 0
-    for i in range(n):
+    launches = [0]
+
+    def call(name, fn, *args):
         if timers is not None:
-            timers.start("axpy")
-        es.es_perturb(plan, int(seeds[i]), sigma, stream)
-        # (rollout of the perturbed model happens here; its reward is an input)
-        es.es_restore(plan, int(seeds[i]), sigma, stream)
+            timers.start(name)
+        fn(*args)
         if timers is not None:
-            timers.stop("axpy", 2)
-        launches += 2
+            timers.stop(name, 1)
+        launches[0] += 1
+
+    # (the rollout of each perturbed model happens after its perturb; its
+    # reward is an input here)
+    if fused:
+        call("perturb", es.es_perturb, plan, int(seeds[0]), sigma, stream)
+        for i in range(1, n):
+            call("restore_perturb", es.es_restore_perturb, plan, int(seeds[i - 1]), sigma,
+                 int(seeds[i]), sigma, stream)
+        call("restore", es.es_restore, plan, int(seeds[n - 1]), sigma, stream)
+    else:
+        for i in range(n):
+            call("perturb", es.es_perturb, plan, int(seeds[i]), sigma, stream)
+            call("restore", es.es_restore, plan, int(seeds[i]), sigma, stream)
     rhat = es.es_normalize_rewards(rewards, 1e-8)
     coeffs = es.es_update_coeffs(rhat, wl.alpha, sigma, es.ES_SCALE_PAPER)
-    if timers is not None:
-        timers.start("update")
-    es.es_update(plan, seeds, coeffs, stream)
-    if timers is not None:
-        timers.stop("update", 1)
     if np.any(coeffs != 0):
-        launches += 1
-    return launches
+        call("update", es.es_update, plan, seeds, coeffs, stream)
+    else:
+        es.es_update(plan, seeds, coeffs, stream)   # no launch: the no-update rule
+    return launches[0]
 
 
 class KernelTimers:
@@ -199,15 +210,50 @@ class KernelTimers:
         e.record(self.stream)
         self.pairs.setdefault(name, []).append((self._open.pop(name), e, count))
 
+    def names(self):
+        return list(self.pairs)
+
+    def count(self, name):
+        return sum(c for _, _, c in self.pairs.get(name, []))
+
     def mean_ms(self, name):
-        tot, cnt = 0.0, 0
-        for a, b, c in self.pairs.get(name, []):
-            tot += a.elapsed_time(b)
-            cnt += c
-        return tot / cnt if cnt else None
+        cnt = self.count(name)
+        return self.total_ms(name) / cnt if cnt else None
 
     def total_ms(self, name):
         return sum(a.elapsed_time(b) for a, b, _ in self.pairs.get(name, []))
+
+
+# Gaussians each launch kind draws per parameter (the update draws N).
+GAUSS_PER_ELEM = {"perturb": 1, "restore": 1, "restore_perturb": 2}
+KERNEL_NAME = {"perturb": "axpy_noise_kernel<1 step> (es_perturb)",
+               "restore": "axpy_noise_kernel<1 step> (es_restore)",
+               "restore_perturb": "axpy_noise_kernel<2 steps> (es_restore_perturb)",
+               "update": "update_kernel (es_update)"}
+# Philox4x32-10: 10 rounds x 2 products of 32x32->64 bits per 4 outputs, each
+# product two 32-bit multiplies (high and low word): 10 per Gaussian.
+IMUL_PER_GAUSS = 10
+IMUL_PER_CLK_SM = 64
+
+
+def traffic_per_element(kind):
+    """DRAM bytes per parameter of one launch from the committed ncu summary,
+    or None if the kernel sources changed since that capture."""
+    import hashlib
+    path = os.path.join(ROOT, "profiles", "dram_traffic.txt")
+    if not os.path.exists(path):
+        return None
+    h = hashlib.sha256()
+    csrc = os.path.join(ROOT, "paper_2608_17310_gb300", "csrc")
+    for f in sorted(os.listdir(csrc)):
+        with open(os.path.join(csrc, f), "rb") as fh:
+            h.update(fh.read())
+    digest = h.hexdigest()[:16]
+    for line in open(path):
+        f = line.split()
+        if len(f) == 3 and not line.startswith("#") and f[0] == kind:
+            return float(f[1]) if f[2] == digest else None
+    return None
 
 
 def run_ours(args, rank, world, dist):
@@ -239,6 +285,7 @@ def run_ours(args, rank, world, dist):
     torch.cuda.synchronize()
 
     timers = KernelTimers(torch, stream)
+    fused = not args.unfused
     launches = 0
     ev0 = torch.cuda.Event(enable_timing=True)
     ev1 = torch.cuda.Event(enable_timing=True)
@@ -246,7 +293,7 @@ def run_ours(args, rank, world, dist):
         ev0.record(stream)
         for k in range(args.steps):
             t = args.warmup + k
-            launches += run_step(es, plan, wl, t, n, sigma_at(t), s_handle, timers)
+            launches += run_step(es, plan, wl, t, n, sigma_at(t), s_handle, timers, fused)
         ev1.record(stream)
         torch.cuda.synchronize()
     barrier(dist)
@@ -256,17 +303,44 @@ def run_ours(args, rank, world, dist):
     per_step_ms = ms_max / args.steps
     value = world * P * n * args.steps / (ms_max / 1e3)
 
-    axpy_ms = timers.mean_ms("axpy")
-    upd_ms = timers.mean_ms("update")
     hbm_gbs, sm_max_mhz, peak_src = peaks()
-    axpy_bytes = 2 * esize * P
-    axpy_gbs = axpy_bytes / (axpy_ms / 1e3) / 1e9
-    axpy_share = timers.total_ms("axpy") / ms
-    upd_share = timers.total_ms("update") / ms
+    sms = torch.cuda.get_device_properties(dev_index).multi_processor_count
+    imul_peak = sms * IMUL_PER_CLK_SM * sm_max_mhz * 1e6          # 32-bit multiplies / s
+    gauss_peak = imul_peak / IMUL_PER_GAUSS
+    bytes_per_launch = 2 * esize * P
+    kernels = {}
+    for name in timers.names():
+        mean = timers.mean_ms(name)
+        g = GAUSS_PER_ELEM.get(name, n) * P
+        gbs = bytes_per_launch / (mean / 1e3) / 1e9
+        gps = g / (mean / 1e3)
+        hbm_frac, alu_frac = gbs / hbm_gbs, gps / gauss_peak
+        kernels[name] = {"kernel": KERNEL_NAME[name], "launches": timers.count(name),
+                         "mean_ms": mean, "share": timers.total_ms(name) / ms,
+                         "gbs": gbs, "gauss_per_s": gps, "hbm_frac": hbm_frac,
+                         "alu_frac": alu_frac, "bound": "alu" if alu_frac > hbm_frac else "hbm"}
+    dom = max(kernels, key=lambda k: kernels[k]["share"])
+    d = kernels[dom]
+    tpe = traffic_per_element(dom)
+    traffic = tpe * P if tpe is not None else None
+    if d["bound"] == "hbm":
+        roof = {"bound": "hbm", "achieved": d["gbs"], "peak": hbm_gbs, "unit": "GB/s",
+                "frac": d["hbm_frac"], "traffic": traffic,
+                "peak_source": f"{peak_src} MEASURED_PEAKS.json hbm_gbs"}
+    else:
+        roof = {"bound": "alu", "achieved": d["gauss_per_s"] * IMUL_PER_GAUSS / 1e12,
+                "peak": imul_peak / 1e12, "unit": "T imul32/s", "frac": d["alu_frac"],
+                "traffic": traffic,
+                "peak_source": f"{sms} SMs x {IMUL_PER_CLK_SM} 32-bit integer multiplies/clk x "
+                               f"{sm_max_mhz:.0f} MHz; {IMUL_PER_GAUSS} multiplies per Gaussian"}
+    roof.update({"kernel": d["kernel"], "hbm_frac": d["hbm_frac"], "alu_frac": d["alu_frac"],
+                 "algorithmic_bytes_per_launch": bytes_per_launch,
+                 "gaussians_per_launch": GAUSS_PER_ELEM.get(dom, n) * P})
 
     e2e = None
     if not args.no_e2e:
-        e2e = run_e2e(args, torch, es, plan, params, wl, n, esize, sigma_at, s_handle, dist, world)
+        e2e = run_e2e(args, torch, es, plan, params, wl, n, esize, sigma_at, s_handle, dist, world,
+                      fused)
 
     cpu = None
     if not args.no_cpu_baseline and rank == 0 and world == 1:
@@ -276,23 +350,16 @@ def run_ours(args, rank, world, dist):
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": per_step_ms,
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
-        "dtype": wl.dtype, "data": "synthetic",
+        "dtype": "f32", "data": "synthetic",
         "config": {"workload": args.workload, "params": P, "population": n,
+                   "storage": wl.dtype,
                    "segments": len(specs), "description": wl.description,
                    "sigma": sigma_at(args.warmup), "alpha": wl.alpha,
+                   "generation_loop": "fused es_restore_perturb" if fused else "separate calls",
                    "l2": "inputs larger than L2 (%.1f GB of parameters)" % (P * esize / 1e9),
                    "parallelism": "replicas" if world > 1 else "single GPU"},
-        "roofline": {"bound": "hbm", "achieved": axpy_gbs, "peak": hbm_gbs, "unit": "GB/s",
-                     "frac": axpy_gbs / hbm_gbs, "traffic": None,
-                     "kernel": "axpy_noise_kernel<Bf16Io> (es_perturb / es_restore)",
-                     "peak_source": f"{peak_src} MEASURED_PEAKS.json hbm_gbs"},
-        "kernels": {
-            "axpy_noise": {"mean_ms": axpy_ms, "share": axpy_share,
-                           "gbs": axpy_gbs, "gauss_per_s": P / (axpy_ms / 1e3)},
-            "update": {"mean_ms": upd_ms, "share": upd_share,
-                       "gauss_per_s": P * n / (upd_ms / 1e3) if upd_ms else None,
-                       "gbs": axpy_bytes / (upd_ms / 1e3) / 1e9 if upd_ms else None},
-        },
+        "roofline": roof,
+        "kernels": kernels,
         "gpu_launches": launches,
         "clocks": clk.summary(),
         "e2e": e2e,
@@ -303,7 +370,7 @@ def run_ours(args, rank, world, dist):
         print(json.dumps(out), flush=True)
 
 
-def run_e2e(args, torch, es, plan, params, wl, n, esize, sigma_at, s_handle, dist, world):
+def run_e2e(args, torch, es, plan, params, wl, n, esize, sigma_at, s_handle, dist, world, fused):
     """Same step with the parameters in pinned host memory: H2D copy, step, D2H copy."""
     host = [torch.empty(p.shape, dtype=p.dtype, pin_memory=True) for p in params]
     for h, p in zip(host, params):
@@ -314,7 +381,7 @@ def run_e2e(args, torch, es, plan, params, wl, n, esize, sigma_at, s_handle, dis
     def one(t):
         for h, p in zip(host, params):
             p.copy_(h, non_blocking=True)
-        launches = run_step(es, plan, wl, t, n, sigma_at(t), s_handle)
+        launches = run_step(es, plan, wl, t, n, sigma_at(t), s_handle, None, fused)
         for h, p in zip(host, params):
             h.copy_(p, non_blocking=True)
         return launches
@@ -390,7 +457,7 @@ def run_reference(args, rank, world, dist):
     out = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world,
            "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * tot / args.steps,
            "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
-           "dtype": wl.dtype, "data": "synthetic", "impl": "reference",
+           "dtype": "f64", "data": "synthetic", "impl": "reference",
            "config": {"workload": args.workload, "population": n, "sample_params": m},
            "cpu_baseline": {"value": value, "unit": UNIT, "cores": 1, "kind": "oracle",
                             "sample": desc},

@@ -186,6 +186,21 @@ es_status_t es_perturb(es_plan_t plan, uint64_t seed, float sigma, void* stream)
 es_status_t es_restore(es_plan_t plan, uint64_t seed, float sigma, void* stream);
 
 /*
+ * Restore one member and perturb the next in a single pass over theta:
+ *   theta[g] <- round(round(theta[g] - sigma_restore * eps_{restore_seed}[g])
+ *                     + sigma_perturb * eps_{perturb_seed}[g]),
+ * bit-identical to es_restore(plan, restore_seed, sigma_restore) followed by
+ * es_perturb(plan, perturb_seed, sigma_perturb): the intermediate value is
+ * rounded to the storage type exactly as the separate calls would store it.
+ * In the generation loop of §3 / App. D.6 the restore of member i and the
+ * perturb of member i + 1 are adjacent (the next rollout follows the
+ * perturb), so this halves the passes over the parameters in that loop.
+ * Errors as es_perturb.
+ */
+es_status_t es_restore_perturb(es_plan_t plan, uint64_t restore_seed, float sigma_restore,
+                               uint64_t perturb_seed, float sigma_perturb, void* stream);
+
+/*
  * Fused reward-weighted update over the whole population in one pass (§3
  * implemented update; App. C.1):
  *   theta[g] <- round(theta[g] + sum_{i=0}^{n-1} coeffs[i] * eps_{seeds[i]}[g]),

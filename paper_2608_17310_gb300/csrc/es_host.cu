@@ -248,6 +248,20 @@ es_status_t es_restore(es_plan_t plan, uint64_t seed, float sigma, void* stream)
   return axpy(plan, seed, -sigma, stream, "es_restore");
 }
 
+es_status_t es_restore_perturb(es_plan_t plan, uint64_t restore_seed, float sigma_restore,
+                               uint64_t perturb_seed, float sigma_perturb, void* stream) {
+  if (plan == nullptr) return fail(ES_ERR_INVALID_ARG, "es_restore_perturb: plan is NULL");
+  if (!std::isfinite(sigma_restore) || !std::isfinite(sigma_perturb))
+    return fail(ES_ERR_NONFINITE, "es_restore_perturb: sigma is not finite");
+  es_status_t st = check_plan_device(plan);
+  if (st != ES_OK) return st;
+  cudaError_t err = esopt::launch_axpy_noise2(view(plan), restore_seed, -sigma_restore,
+                                              perturb_seed, sigma_perturb,
+                                              static_cast<cudaStream_t>(stream));
+  if (err != cudaSuccess) return cuda_fail(err, "es_restore_perturb");
+  return ok();
+}
+
 es_status_t es_update(es_plan_t plan, const uint64_t* seeds, const float* coeffs, int n,
                       void* stream) {
   if (plan == nullptr) return fail(ES_ERR_INVALID_ARG, "es_update: plan is NULL");

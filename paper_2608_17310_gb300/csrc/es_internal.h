@@ -50,6 +50,8 @@ struct PlanView {
 // Kernel launchers (es_kernels.cu). Each returns the launch's cudaError_t.
 cudaError_t launch_axpy_noise(const PlanView& plan, uint64_t seed, float scale,
                               cudaStream_t stream);
+cudaError_t launch_axpy_noise2(const PlanView& plan, uint64_t seed, float scale, uint64_t seed2,
+                               float scale2, cudaStream_t stream);
 cudaError_t launch_update(const PlanView& plan, const UpdateArgs& args,
                           cudaStream_t stream);
 cudaError_t launch_noise_bits(uint64_t seed, uint64_t block_base, uint64_t nblocks,

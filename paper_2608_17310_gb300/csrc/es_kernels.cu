@@ -38,6 +38,16 @@ struct Bf16Io {
   __device__ static uint4 pack(const float (&f)[8]) {
     return make_uint4(pack2(f[0], f[1]), pack2(f[2], f[3]), pack2(f[4], f[5]), pack2(f[6], f[7]));
   }
+  // f <- value of round_to_storage(f), element-wise (one rounding to bf16).
+  __device__ static void round_trip(float (&f)[8]) {
+#pragma unroll
+    for (int k = 0; k < 8; k += 2) {
+      const uint32_t w = pack2(f[k], f[k + 1]);
+      f[k] = __uint_as_float(w << 16);
+      f[k + 1] = __uint_as_float(w & 0xFFFF0000u);
+    }
+  }
+  __device__ static float round_trip1(float f) { return to_f32(from_f32(f)); }
   // Gaussians of the 8 elements starting at global index g0 (g0 % 8 == 0).
   __device__ static void noise(uint64_t g0, PhiloxKey key, float (&e)[8]) {
     const uint64_t j = g0 >> 2;
@@ -61,6 +71,8 @@ struct F32Io {
     return make_uint4(__float_as_uint(f[0]), __float_as_uint(f[1]),
                       __float_as_uint(f[2]), __float_as_uint(f[3]));
   }
+  __device__ static void round_trip(float (&)[4]) {}
+  __device__ static float round_trip1(float f) { return f; }
   __device__ static void noise(uint64_t g0, PhiloxKey key, float (&e)[4]) {
     const float4 a = gaussian4(g0 >> 2, key);
     e[0] = a.x; e[1] = a.y; e[2] = a.z; e[3] = a.w;
@@ -74,11 +86,15 @@ __device__ __forceinline__ const SegDesc* find_segment(const SegDesc* __restrict
   return segs + seg;
 }
 
-// theta[g] <- round(theta[g] + scale * eps_seed[g]) over every segment.
-template <class Io>
+// theta[g] <- round(theta[g] + scale * eps_seed[g]) over every segment; with
+// kTwo, a second step round(. + scale2 * eps_seed2[g]) follows in registers,
+// after the first result has been rounded to the storage type exactly as a
+// separate launch would store it (restore of one member fused with the
+// perturb of the next).
+template <class Io, bool kTwo>
 __global__ void __launch_bounds__(kBlockThreads)
 axpy_noise_kernel(const SegDesc* __restrict__ segs, uint64_t total_tiles, PhiloxKey key,
-                  float scale) {
+                  float scale, PhiloxKey key2, float scale2) {
   constexpr int V = Io::kVec;
   constexpr uint64_t kTile = static_cast<uint64_t>(kBlockThreads) * kVecsPerThread * V;
   using S = typename Io::Scalar;
@@ -107,12 +123,27 @@ axpy_noise_kernel(const SegDesc* __restrict__ segs, uint64_t total_tiles, Philox
         Io::unpack(v[u], f);
 #pragma unroll
         for (int k = 0; k < V; ++k) f[k] = fmaf(scale, eps[k], f[k]);
+        if (kTwo) {
+          Io::round_trip(f);
+          Io::noise(index_base + e, key2, eps);
+#pragma unroll
+          for (int k = 0; k < V; ++k) f[k] = fmaf(scale2, eps[k], f[k]);
+        }
         *reinterpret_cast<uint4*>(base + e) = Io::pack(f);
       } else {  // ragged end of a segment
         const int rem = static_cast<int>(numel - e);
+        float f[V];
 #pragma unroll
         for (int k = 0; k < V; ++k)
-          if (k < rem) base[e + k] = Io::from_f32(fmaf(scale, eps[k], Io::to_f32(base[e + k])));
+          f[k] = k < rem ? fmaf(scale, eps[k], Io::to_f32(base[e + k])) : 0.0f;
+        if (kTwo) {
+          Io::noise(index_base + e, key2, eps);
+#pragma unroll
+          for (int k = 0; k < V; ++k) f[k] = fmaf(scale2, eps[k], Io::round_trip1(f[k]));
+        }
+#pragma unroll
+        for (int k = 0; k < V; ++k)
+          if (k < rem) base[e + k] = Io::from_f32(f[k]);
       }
     }
   }
@@ -246,21 +277,31 @@ int persistent_grid(K kernel, uint64_t work_items) {
   return grid < 1 ? 1 : static_cast<int>(grid);
 }
 
+template <bool kTwo>
+cudaError_t launch_axpy(const PlanView& plan, PhiloxKey key, float scale, PhiloxKey key2,
+                        float scale2, cudaStream_t stream) {
+  if (plan.dtype == ES_BF16) {
+    auto k = axpy_noise_kernel<Bf16Io, kTwo>;
+    k<<<persistent_grid(k, plan.total_tiles), kBlockThreads, 0, stream>>>(
+        plan.segs, plan.total_tiles, key, scale, key2, scale2);
+  } else {
+    auto k = axpy_noise_kernel<F32Io, kTwo>;
+    k<<<persistent_grid(k, plan.total_tiles), kBlockThreads, 0, stream>>>(
+        plan.segs, plan.total_tiles, key, scale, key2, scale2);
+  }
+  return cudaGetLastError();
+}
+
 }  // namespace
 
 cudaError_t launch_axpy_noise(const PlanView& plan, uint64_t seed, float scale,
                               cudaStream_t stream) {
-  const PhiloxKey key = philox_key(seed);
-  if (plan.dtype == ES_BF16) {
-    auto k = axpy_noise_kernel<Bf16Io>;
-    k<<<persistent_grid(k, plan.total_tiles), kBlockThreads, 0, stream>>>(
-        plan.segs, plan.total_tiles, key, scale);
-  } else {
-    auto k = axpy_noise_kernel<F32Io>;
-    k<<<persistent_grid(k, plan.total_tiles), kBlockThreads, 0, stream>>>(
-        plan.segs, plan.total_tiles, key, scale);
-  }
-  return cudaGetLastError();
+  return launch_axpy<false>(plan, philox_key(seed), scale, PhiloxKey{0u, 0u}, 0.0f, stream);
+}
+
+cudaError_t launch_axpy_noise2(const PlanView& plan, uint64_t seed, float scale, uint64_t seed2,
+                               float scale2, cudaStream_t stream) {
+  return launch_axpy<true>(plan, philox_key(seed), scale, philox_key(seed2), scale2, stream);
 }
 
 cudaError_t launch_update(const PlanView& plan, const UpdateArgs& args, cudaStream_t stream) {

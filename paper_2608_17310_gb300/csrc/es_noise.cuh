@@ -75,11 +75,22 @@ __device__ __forceinline__ float sqrt_approx(float x) {
   return r;
 }
 
+// radius^2 = -2 ln u for u = uniform_open(x), fast path:
+//   for u <= 1 - 2^-10: -2 ln 2 * log2(u) with the MUFU log2 (__log2f);
+//   for u >  1 - 2^-10: 2t + t^2 + (2/3) t^3 with t = 1 - u (exact), whose
+//     truncation error is below t^3/4 relative (an absolute log2 error there
+//     would be a large relative error of the small radius).
+// Both are evaluated and one is selected, which keeps the code free of
+// divergent branches.
+__device__ __forceinline__ float radius_sq(float u) {
+  const float t = 1.0f - u;
+  const float series = t * fmaf(t, fmaf(t, 2.0f / 3.0f, 1.0f), 2.0f);
+  const float logged = __log2f(u) * kMinusTwoLn2;
+  return u > kNearOne ? series : logged;
+}
+
 // One Box-Muller pair, fast path:
-//   radius^2 = -2 ln u_a:  for u_a <= 1 - 2^-10, -2 ln 2 * log2(u_a) with the
-//     MUFU log2 (__log2f); for u_a > 1 - 2^-10, 2t + t^2 + (2/3) t^3 with
-//     t = 1 - u_a (exact), whose truncation error is below t^3/4 relative;
-//   radius = sqrt.approx(radius^2);
+//   radius = sqrt.approx(radius_sq(u_a));
 //   angle: 2 pi u_b = 2 pi s + pi with s = u_b - 1/2 formed exactly from the
 //     bits, so cos/sin of 2 pi u_b are -cos/-sin of 2 pi s, an argument in
 //     (-pi, pi) where __sincosf is accurate.
@@ -87,15 +98,7 @@ __device__ __forceinline__ float sqrt_approx(float x) {
 // (every 23-bit radius input and every 23-bit angle input) by the test suite;
 // the error stays below 1e-5 * max(1, |eps|).
 __device__ __forceinline__ float2 box_muller(uint32_t xa, uint32_t xb) {
-  const float ua = uniform_open(xa);
-  float r2;
-  if (ua > kNearOne) {
-    const float t = 1.0f - ua;
-    r2 = t * fmaf(t, fmaf(t, 2.0f / 3.0f, 1.0f), 2.0f);
-  } else {
-    r2 = __log2f(ua) * kMinusTwoLn2;
-  }
-  const float r = sqrt_approx(r2);
+  const float r = sqrt_approx(radius_sq(uniform_open(xa)));
   const float s = (__uint_as_float(0x3F800000u | (xb >> 9)) - 1.5f) + 0x1p-24f;
   float sn, cs;
   __sincosf(s * kTwoPi, &sn, &cs);

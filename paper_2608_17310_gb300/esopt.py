@@ -80,6 +80,7 @@ def _load() -> ctypes.CDLL:
         "es_box_muller": (i32, [vp, u64, vp, vp]),
         "es_perturb": (i32, [vp, u64, f32, vp]),
         "es_restore": (i32, [vp, u64, f32, vp]),
+        "es_restore_perturb": (i32, [vp, u64, f32, u64, f32, vp]),
         "es_update": (i32, [vp, P(u64), P(f32), i32, vp]),
         "es_normalize_rewards": (i32, [P(f64), i32, f64, P(f64)]),
         "es_sigma_cosine": (f64, [f64, f64, i32, i32]),
@@ -254,6 +255,12 @@ def es_perturb(plan: Plan, seed: int, sigma: float, stream=None) -> None:
 
 def es_restore(plan: Plan, seed: int, sigma: float, stream=None) -> None:
     _check(_load().es_restore(plan.handle, seed, sigma, _stream(stream)), "es_restore")
+
+
+def es_restore_perturb(plan: Plan, restore_seed: int, sigma_restore: float, perturb_seed: int,
+                       sigma_perturb: float, stream=None) -> None:
+    _check(_load().es_restore_perturb(plan.handle, restore_seed, sigma_restore, perturb_seed,
+                                      sigma_perturb, _stream(stream)), "es_restore_perturb")
 
 
 def es_update(plan: Plan, seeds, coeffs, stream=None) -> None:

@@ -93,6 +93,37 @@ def test_perturb_then_restore_match_oracle(es, oracle, dtype, layout):
 
 
 @pytest.mark.parametrize("dtype", ["bf16", "f32"])
+def test_restore_perturb_is_bit_identical_to_the_two_calls(es, oracle, dtype):
+    a = make_params(dtype, RAGGED, seed=7)
+    b = [t.clone() for t in a]
+    plan_a, segs = build_plan(es, a, _sparse64(len(RAGGED)))
+    plan_b, _ = build_plan(es, b, _sparse64(len(RAGGED)))
+    s1, s2, sig1, sig2 = 11, 2**45 + 3, 1e-3, 7e-4
+    for p in (plan_a, plan_b):
+        es.es_perturb(p, s1, sig1)
+    torch.cuda.synchronize()
+    mid = [host_values(t) for t in a]
+    es.es_restore(plan_a, s1, sig1)
+    es.es_perturb(plan_a, s2, sig2)
+    es.es_restore_perturb(plan_b, s1, sig1, s2, sig2)
+    torch.cuda.synchronize()
+    iv = torch.int16 if dtype == "bf16" else torch.int32
+    for x, y in zip(a, b):
+        assert torch.equal(x.view(iv), y.view(iv))
+    # and against the oracle, step by step
+    g = indices(segs)
+    for k in range(len(a)):
+        want = oracle.perturb(oracle.restore(mid[k], g[k], s1, sig1, dtype), g[k], s2, sig2, dtype)
+        tol = noise_abs_tol([oracle.noise_at(s1, g[k]), oracle.noise_at(s2, g[k])], [sig1, sig2])
+        compare(dtype, host_values(b[k]), want, f"restore+perturb seg {k}", tol)
+    with pytest.raises(es.EsError) as ei:
+        es.es_restore_perturb(plan_b, 1, float("nan"), 2, 1e-3)
+    assert ei.value.status == es.ES_ERR_NONFINITE
+    plan_a.close()
+    plan_b.close()
+
+
+@pytest.mark.parametrize("dtype", ["bf16", "f32"])
 @pytest.mark.parametrize("nseeds", [1, 2, 3, 8, 30, 129, 256])
 def test_update_matches_oracle(es, oracle, dtype, nseeds):
     numels = [9, 8193, 20000, 4096 * 3 + 5]
