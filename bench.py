@@ -150,6 +150,18 @@ class ClockSampler:
 
 # --- the step -------------------------------------------------------------------------------
 
+def workload_config(workload: str, n: int, world: int) -> dict:
+    """The `config` object of the JSON line (shared by both arms)."""
+    wl = I.WORKLOADS[workload]
+    specs = I.shapes_for(workload)
+    P = sum(s.numel for s in specs)
+    esize = 2 if wl.dtype == "bf16" else 4
+    return {"workload": workload, "params": P, "population": n, "storage": wl.dtype,
+            "segments": len(specs), "description": wl.description, "alpha": wl.alpha,
+            "l2": "inputs larger than L2 (%.1f GB of parameters)" % (P * esize / 1e9),
+            "parallelism": "replicas" if world > 1 else "single GPU"}
+
+
 def generation_inputs(wl, step: int, n: int):
     """Seeds and rewards of one generation (rewards stand in for rollouts)."""
     seeds = I.population_seeds(n, generation=step)
@@ -351,13 +363,8 @@ def run_ours(args, rank, world, dist):
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": per_step_ms,
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
         "dtype": "f32", "data": "synthetic",
-        "config": {"workload": args.workload, "params": P, "population": n,
-                   "storage": wl.dtype,
-                   "segments": len(specs), "description": wl.description,
-                   "sigma": sigma_at(args.warmup), "alpha": wl.alpha,
-                   "generation_loop": "fused es_restore_perturb" if fused else "separate calls",
-                   "l2": "inputs larger than L2 (%.1f GB of parameters)" % (P * esize / 1e9),
-                   "parallelism": "replicas" if world > 1 else "single GPU"},
+        "config": dict(workload_config(args.workload, n, world), sigma=sigma_at(args.warmup),
+                       generation_loop="fused es_restore_perturb" if fused else "separate calls"),
         "roofline": roof,
         "kernels": kernels,
         "gpu_launches": launches,
@@ -458,7 +465,7 @@ def run_reference(args, rank, world, dist):
            "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * tot / args.steps,
            "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
            "dtype": "f64", "data": "synthetic", "impl": "reference",
-           "config": {"workload": args.workload, "population": n, "sample_params": m},
+           "config": dict(workload_config(args.workload, n, 1), sigma=sigma, sample_params=m),
            "cpu_baseline": {"value": value, "unit": UNIT, "cores": 1, "kind": "oracle",
                             "sample": desc},
            "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0,

@@ -56,8 +56,9 @@
 extern "C" {
 #endif
 
-/* Largest population (number of seeds) one es_update call accepts. */
-#define ES_MAX_SEEDS 256
+/* Largest population (number of seeds) one es_update call accepts, and the
+   largest number of seeds one generation of es_replay may have. */
+#define ES_MAX_SEEDS 1024
 
 typedef enum {
   ES_OK = 0,
@@ -192,6 +193,8 @@ es_status_t es_restore(es_plan_t plan, uint64_t seed, float sigma, void* stream)
  * bit-identical to es_restore(plan, restore_seed, sigma_restore) followed by
  * es_perturb(plan, perturb_seed, sigma_perturb): the intermediate value is
  * rounded to the storage type exactly as the separate calls would store it.
+ * With restore_seed == perturb_seed (the two members of an antithetic pair,
+ * sigma_perturb = -sigma_restore) the noise is generated once.
  * In the generation loop of §3 / App. D.6 the restore of member i and the
  * perturb of member i + 1 are adjacent (the next rollout follows the
  * perturb), so this halves the passes over the parameters in that loop.
@@ -214,6 +217,36 @@ es_status_t es_restore_perturb(es_plan_t plan, uint64_t restore_seed, float sigm
  */
 es_status_t es_update(es_plan_t plan, const uint64_t* seeds, const float* coeffs,
                       int n, void* stream);
+
+/*
+ * The update of one generation fused with the first perturb of the next:
+ *   theta[g] <- round(round(theta[g] + sum_i coeffs[i] * eps_{seeds[i]}[g])
+ *                     + sigma_next * eps_{next_seed}[g]),
+ * bit-identical to es_update(plan, seeds, coeffs, n) followed by
+ * es_perturb(plan, next_seed, sigma_next), in one pass over theta. If every
+ * coefficient is 0 this is es_perturb alone. Errors as es_update, and
+ * ES_ERR_NONFINITE for sigma_next.
+ */
+es_status_t es_update_perturb(es_plan_t plan, const uint64_t* seeds, const float* coeffs,
+                              int n, uint64_t next_seed, float sigma_next, void* stream);
+
+/*
+ * Replay of a logged run: the paper records the seed of every update and, for
+ * evaluation, reloads the base checkpoint and reconstructs the update sequence
+ * deterministically from those seeds (App. D.2, D.3, D.4). For g = 0 ..
+ * generations-1, in order:
+ *   theta[g] <- round(theta[g] + sum_{i in generation g} coeffs[i] * eps_{seeds[i]}[g]),
+ * bit-identical to one es_update per generation. `seeds` and `coeffs` hold
+ * the generations back to back; counts[g] (1 .. ES_MAX_SEEDS) is the size of
+ * generation g. Up to 256 generations and ES_MAX_SEEDS seeds are fused per
+ * pass over theta; longer logs take several passes, split between
+ * generations. Host arrays; asynchronous on `stream`.
+ * Errors: ES_ERR_INVALID_ARG (NULL, generations < 1, an empty generation),
+ * ES_ERR_TOO_MANY_SEEDS (a generation over ES_MAX_SEEDS), ES_ERR_NONFINITE,
+ * ES_ERR_WRONG_DEVICE, ES_ERR_CUDA.
+ */
+es_status_t es_replay(es_plan_t plan, const uint64_t* seeds, const float* coeffs,
+                      const int* counts, int generations, void* stream);
 
 /*
  * Population z-score of the rewards (§3):

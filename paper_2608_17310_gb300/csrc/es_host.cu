@@ -61,6 +61,51 @@ esopt::PlanView view(const es_plan* plan) {
   return esopt::PlanView{plan->d_segs, plan->total_tiles, plan->dtype};
 }
 
+es_status_t check_update_inputs(es_plan_t plan, const uint64_t* seeds, const float* coeffs, int n,
+                                const char* what) {
+  if (plan == nullptr) return fail(ES_ERR_INVALID_ARG, "%s: plan is NULL", what);
+  if (seeds == nullptr || coeffs == nullptr || n < 1)
+    return fail(ES_ERR_INVALID_ARG, "%s: need n >= 1 seeds and coefficients", what);
+  if (n > ES_MAX_SEEDS)
+    return fail(ES_ERR_TOO_MANY_SEEDS, "%s: n = %d > ES_MAX_SEEDS = %d", what, n, ES_MAX_SEEDS);
+  for (int i = 0; i < n; ++i)
+    if (!std::isfinite(coeffs[i]))
+      return fail(ES_ERR_NONFINITE, "%s: coefficient %d is not finite", what, i);
+  return check_plan_device(plan);
+}
+
+void start_update(esopt::UpdateArgs& a) {
+  a.n = 0;
+  a.n_gen = 0;
+  a.perturb = 0;
+  a.pscale = 0.0f;
+  a.pkey[0] = a.pkey[1] = 0u;
+}
+
+// Appends one generation, skipping seeds whose coefficient is 0 (they add
+// exactly zero); a generation left empty is dropped, since theta + 0 rounds to
+// theta. The caller guarantees the space.
+void append_generation(esopt::UpdateArgs& a, const uint64_t* seeds, const float* coeffs,
+                       int count) {
+  const int before = a.n;
+  for (int i = 0; i < count; ++i) {
+    if (coeffs[i] == 0.0f) continue;
+    const esopt::PhiloxKey key = esopt::philox_key(seeds[i]);
+    a.key[a.n][0] = key.k0;
+    a.key[a.n][1] = key.k1;
+    a.coeff[a.n] = coeffs[i];
+    ++a.n;
+  }
+  if (a.n > before) a.gen_end[a.n_gen++] = static_cast<uint16_t>(a.n);
+}
+
+es_status_t launch_update_args(es_plan_t plan, const esopt::UpdateArgs& args, void* stream,
+                               const char* what) {
+  cudaError_t err = esopt::launch_update(view(plan), args, static_cast<cudaStream_t>(stream));
+  if (err != cudaSuccess) return cuda_fail(err, what);
+  return ok();
+}
+
 es_status_t axpy(es_plan_t plan, uint64_t seed, float scale, void* stream, const char* what) {
   if (plan == nullptr) return fail(ES_ERR_INVALID_ARG, "%s: plan is NULL", what);
   if (!std::isfinite(scale)) return fail(ES_ERR_NONFINITE, "%s: sigma is not finite", what);
@@ -264,30 +309,72 @@ es_status_t es_restore_perturb(es_plan_t plan, uint64_t restore_seed, float sigm
 
 es_status_t es_update(es_plan_t plan, const uint64_t* seeds, const float* coeffs, int n,
                       void* stream) {
-  if (plan == nullptr) return fail(ES_ERR_INVALID_ARG, "es_update: plan is NULL");
-  if (seeds == nullptr || coeffs == nullptr || n < 1)
-    return fail(ES_ERR_INVALID_ARG, "es_update: need n >= 1 seeds and coefficients");
-  if (n > ES_MAX_SEEDS)
-    return fail(ES_ERR_TOO_MANY_SEEDS, "es_update: n = %d > ES_MAX_SEEDS = %d", n, ES_MAX_SEEDS);
+  es_status_t st = check_update_inputs(plan, seeds, coeffs, n, "es_update");
+  if (st != ES_OK) return st;
   esopt::UpdateArgs args;
-  std::memset(&args, 0, sizeof args);
-  int m = 0;
-  for (int i = 0; i < n; ++i) {
-    if (!std::isfinite(coeffs[i]))
-      return fail(ES_ERR_NONFINITE, "es_update: coefficient %d is not finite", i);
-    if (coeffs[i] == 0.0f) continue;  // adds exactly zero to every accumulator
-    const esopt::PhiloxKey key = esopt::philox_key(seeds[i]);
-    args.key[m][0] = key.k0;
-    args.key[m][1] = key.k1;
-    args.coeff[m] = coeffs[i];
-    ++m;
+  start_update(args);
+  append_generation(args, seeds, coeffs, n);
+  if (args.n_gen == 0) return ok();  // every coefficient 0: no update, theta bit-identical
+  return launch_update_args(plan, args, stream, "es_update");
+}
+
+es_status_t es_update_perturb(es_plan_t plan, const uint64_t* seeds, const float* coeffs, int n,
+                              uint64_t next_seed, float sigma_next, void* stream) {
+  es_status_t st = check_update_inputs(plan, seeds, coeffs, n, "es_update_perturb");
+  if (st != ES_OK) return st;
+  if (!std::isfinite(sigma_next))
+    return fail(ES_ERR_NONFINITE, "es_update_perturb: sigma_next is not finite");
+  esopt::UpdateArgs args;
+  start_update(args);
+  append_generation(args, seeds, coeffs, n);
+  if (args.n_gen == 0) return axpy(plan, next_seed, sigma_next, stream, "es_update_perturb");
+  const esopt::PhiloxKey key = esopt::philox_key(next_seed);
+  args.perturb = 1;
+  args.pkey[0] = key.k0;
+  args.pkey[1] = key.k1;
+  args.pscale = sigma_next;
+  return launch_update_args(plan, args, stream, "es_update_perturb");
+}
+
+es_status_t es_replay(es_plan_t plan, const uint64_t* seeds, const float* coeffs,
+                      const int* counts, int generations, void* stream) {
+  if (plan == nullptr) return fail(ES_ERR_INVALID_ARG, "es_replay: plan is NULL");
+  if (counts == nullptr || generations < 1)
+    return fail(ES_ERR_INVALID_ARG, "es_replay: need at least one generation");
+  uint64_t total = 0;
+  for (int g = 0; g < generations; ++g) {
+    if (counts[g] < 1) return fail(ES_ERR_INVALID_ARG, "es_replay: generation %d is empty", g);
+    if (counts[g] > ES_MAX_SEEDS)
+      return fail(ES_ERR_TOO_MANY_SEEDS, "es_replay: generation %d has %d > ES_MAX_SEEDS = %d seeds",
+                  g, counts[g], ES_MAX_SEEDS);
+    total += static_cast<uint64_t>(counts[g]);
   }
-  if (m == 0) return ok();  // no update: theta stays bit-identical
-  args.n = m;
+  if (seeds == nullptr || coeffs == nullptr)
+    return fail(ES_ERR_INVALID_ARG, "es_replay: NULL seeds or coefficients");
+  for (uint64_t i = 0; i < total; ++i)
+    if (!std::isfinite(coeffs[i]))
+      return fail(ES_ERR_NONFINITE, "es_replay: coefficient %llu is not finite",
+                  static_cast<unsigned long long>(i));
   es_status_t st = check_plan_device(plan);
   if (st != ES_OK) return st;
-  cudaError_t err = esopt::launch_update(view(plan), args, static_cast<cudaStream_t>(stream));
-  if (err != cudaSuccess) return cuda_fail(err, "es_update");
+  // Launches break only between generations, so the roundings are those of
+  // one es_update per generation.
+  esopt::UpdateArgs args;
+  start_update(args);
+  uint64_t off = 0;
+  for (int g = 0; g < generations; ++g) {
+    int nonzero = 0;
+    for (int i = 0; i < counts[g]; ++i) nonzero += coeffs[off + i] != 0.0f;
+    if (nonzero > 0 &&
+        (args.n + nonzero > ES_MAX_SEEDS || args.n_gen == esopt::kMaxGenerations)) {
+      st = launch_update_args(plan, args, stream, "es_replay");
+      if (st != ES_OK) return st;
+      start_update(args);
+    }
+    append_generation(args, seeds + off, coeffs + off, counts[g]);
+    off += static_cast<uint64_t>(counts[g]);
+  }
+  if (args.n_gen > 0) return launch_update_args(plan, args, stream, "es_replay");
   return ok();
 }
 

@@ -12,6 +12,25 @@ namespace esopt {
 
 // Threads per CTA of the streaming kernels.
 constexpr int kBlockThreads = 256;
+// Minimum resident CTAs per SM requested from the compiler (a register cap)
+// for the perturb/restore kernels and for the update kernel; 0 leaves the
+// choice to the compiler.
+#ifndef ES_AXPY_MIN_BLOCKS
+#define ES_AXPY_MIN_BLOCKS 1
+#endif
+#ifndef ES_UPDATE_MIN_BLOCKS
+#define ES_UPDATE_MIN_BLOCKS 0
+#endif
+#if ES_AXPY_MIN_BLOCKS > 0
+#define ES_AXPY_BOUNDS __launch_bounds__(esopt::kBlockThreads, ES_AXPY_MIN_BLOCKS)
+#else
+#define ES_AXPY_BOUNDS __launch_bounds__(esopt::kBlockThreads)
+#endif
+#if ES_UPDATE_MIN_BLOCKS > 0
+#define ES_UPDATE_BOUNDS __launch_bounds__(esopt::kBlockThreads, ES_UPDATE_MIN_BLOCKS)
+#else
+#define ES_UPDATE_BOUNDS __launch_bounds__(esopt::kBlockThreads)
+#endif
 // 16-byte vectors per thread per tile.
 constexpr int kVecsPerThread = 4;
 // Elements per 16-byte vector, per dtype.
@@ -32,14 +51,25 @@ struct SegDesc {
 };
 static_assert(sizeof(SegDesc) == 32, "SegDesc layout");
 
-// Seeds and coefficients of one fused update, passed by value as a kernel
-// parameter and staged in shared memory by each CTA.
+// Largest number of generations one fused update launch applies.
+constexpr int kMaxGenerations = 256;
+
+// One fused update launch: `n_gen` generations of updates, generation g
+// using seeds [gen_end[g-1], gen_end[g]) (gen_end[-1] = 0), each generation
+// rounded to the storage type in turn; then, if `perturb`, one perturb step
+// with (pkey, pscale). Passed by value as a kernel parameter (about 13 KB) and
+// staged in shared memory by each CTA.
 struct UpdateArgs {
-  int n;
-  int pad_;
+  int n;          // seeds in all generations, 1..ES_MAX_SEEDS
+  int n_gen;      // generations, 1..kMaxGenerations
+  int perturb;    // 1: trailing perturb step
+  float pscale;
+  uint32_t pkey[2];
+  uint16_t gen_end[kMaxGenerations];
   uint32_t key[ES_MAX_SEEDS][2];
   float coeff[ES_MAX_SEEDS];
 };
+static_assert(sizeof(UpdateArgs) < 32000, "kernel parameter limit");
 
 struct PlanView {
   const SegDesc* segs;  // device table (nseg + 1 entries)
@@ -51,7 +81,7 @@ struct PlanView {
 cudaError_t launch_axpy_noise(const PlanView& plan, uint64_t seed, float scale,
                               cudaStream_t stream);
 cudaError_t launch_axpy_noise2(const PlanView& plan, uint64_t seed, float scale, uint64_t seed2,
-                               float scale2, cudaStream_t stream);
+                               float scale2, cudaStream_t stream);  // seed2 may equal seed
 cudaError_t launch_update(const PlanView& plan, const UpdateArgs& args,
                           cudaStream_t stream);
 cudaError_t launch_noise_bits(uint64_t seed, uint64_t block_base, uint64_t nblocks,

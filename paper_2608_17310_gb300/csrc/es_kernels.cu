@@ -39,22 +39,29 @@ struct Bf16Io {
     return make_uint4(pack2(f[0], f[1]), pack2(f[2], f[3]), pack2(f[4], f[5]), pack2(f[6], f[7]));
   }
   // f <- value of round_to_storage(f), element-wise (one rounding to bf16).
-  __device__ static void round_trip(float (&f)[8]) {
+  template <int M>
+  __device__ static void round_trip(float (&f)[M]) {
 #pragma unroll
-    for (int k = 0; k < 8; k += 2) {
+    for (int k = 0; k < M; k += 2) {
       const uint32_t w = pack2(f[k], f[k + 1]);
       f[k] = __uint_as_float(w << 16);
       f[k + 1] = __uint_as_float(w & 0xFFFF0000u);
     }
   }
   __device__ static float round_trip1(float f) { return to_f32(from_f32(f)); }
-  // Gaussians of the 8 elements starting at global index g0 (g0 % 8 == 0).
-  __device__ static void noise(uint64_t g0, PhiloxKey key, float (&e)[8]) {
-    const uint64_t j = g0 >> 2;
-    const float4 a = gaussian4(j, key);
-    const float4 b = gaussian4(j + 1, key);
-    e[0] = a.x; e[1] = a.y; e[2] = a.z; e[3] = a.w;
-    e[4] = b.x; e[5] = b.y; e[6] = b.z; e[7] = b.w;
+  // The first `rem` (< 8) elements at base[e], the rest zero, as one vector.
+  __device__ static uint4 load_partial(const uint16_t* base, uint64_t e, int rem) {
+    uint32_t w[4] = {0u, 0u, 0u, 0u};
+#pragma unroll
+    for (int k = 0; k < 8; ++k)
+      if (k < rem) w[k >> 1] |= static_cast<uint32_t>(base[e + k]) << (16 * (k & 1));
+    return make_uint4(w[0], w[1], w[2], w[3]);
+  }
+  __device__ static void store_partial(uint16_t* base, uint64_t e, int rem, const uint4& v) {
+    const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+    for (int k = 0; k < 8; ++k)
+      if (k < rem) base[e + k] = static_cast<uint16_t>(w[k >> 1] >> (16 * (k & 1)));
   }
 };
 
@@ -71,13 +78,82 @@ struct F32Io {
     return make_uint4(__float_as_uint(f[0]), __float_as_uint(f[1]),
                       __float_as_uint(f[2]), __float_as_uint(f[3]));
   }
-  __device__ static void round_trip(float (&)[4]) {}
+  template <int M>
+  __device__ static void round_trip(float (&)[M]) {}
   __device__ static float round_trip1(float f) { return f; }
-  __device__ static void noise(uint64_t g0, PhiloxKey key, float (&e)[4]) {
-    const float4 a = gaussian4(g0 >> 2, key);
-    e[0] = a.x; e[1] = a.y; e[2] = a.z; e[3] = a.w;
+  __device__ static uint4 load_partial(const float* base, uint64_t e, int rem) {
+    uint32_t w[4] = {0u, 0u, 0u, 0u};
+#pragma unroll
+    for (int k = 0; k < 4; ++k)
+      if (k < rem) w[k] = __float_as_uint(base[e + k]);
+    return make_uint4(w[0], w[1], w[2], w[3]);
+  }
+  __device__ static void store_partial(float* base, uint64_t e, int rem, const uint4& v) {
+    const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+    for (int k = 0; k < 4; ++k)
+      if (k < rem) base[e + k] = __uint_as_float(w[k]);
   }
 };
+
+// Philox words of block j for one seed. TileGen serves the blocks of a tile
+// that share the high counter word (per-tile constants, see philox_tile);
+// AnyGen serves any block. Both give the same words.
+struct TileGen {
+  PhiloxTile t;
+  __device__ uint4 block(uint64_t j) const { return philox_block_tile(static_cast<uint32_t>(j), t); }
+};
+struct AnyGen {
+  PhiloxKey key;
+  __device__ uint4 block(uint64_t j) const { return philox_block(j, key); }
+};
+
+template <bool kUniformHi>
+__device__ __forceinline__ auto make_gen(PhiloxKey key, uint32_t j_hi) {
+  if constexpr (kUniformHi) return TileGen{philox_tile(j_hi, key)};
+  else return AnyGen{key};
+}
+
+// f[k] += scale * eps[g0 + k] for the V elements from global index g0
+// (g0 % 4 == 0), with scale folded into each pair's radius.
+template <int V, class Gen>
+__device__ __forceinline__ void add_scaled_noise(const Gen& gen, uint64_t g0, float scale,
+                                                 float (&f)[V]) {
+#pragma unroll
+  for (int b = 0; b < V / 4; ++b) {
+    const uint4 x = gen.block((g0 >> 2) + b);
+    const Polar p = polar(x.x, x.y);
+    const Polar q = polar(x.z, x.w);
+    const float sp = -(scale * p.r), sq = -(scale * q.r);
+    f[4 * b + 0] = fmaf(sp, p.c, f[4 * b + 0]);
+    f[4 * b + 1] = fmaf(sp, p.s, f[4 * b + 1]);
+    f[4 * b + 2] = fmaf(sq, q.c, f[4 * b + 2]);
+    f[4 * b + 3] = fmaf(sq, q.s, f[4 * b + 3]);
+  }
+}
+
+// f <- round(round(f + s1 * eps) + s2 * eps) for one seed's noise, computed
+// once: an antithetic restore (+eps out) followed by the perturb (-eps in).
+template <class Io, int V, class Gen>
+__device__ __forceinline__ void add_scaled_noise_twice(const Gen& gen, uint64_t g0, float s1,
+                                                       float s2, float (&f)[V]) {
+#pragma unroll
+  for (int b = 0; b < V / 4; ++b) {
+    const uint4 x = gen.block((g0 >> 2) + b);
+    const Polar p = polar(x.x, x.y);
+    const Polar q = polar(x.z, x.w);
+    float h[4];
+    h[0] = fmaf(-(s1 * p.r), p.c, f[4 * b + 0]);
+    h[1] = fmaf(-(s1 * p.r), p.s, f[4 * b + 1]);
+    h[2] = fmaf(-(s1 * q.r), q.c, f[4 * b + 2]);
+    h[3] = fmaf(-(s1 * q.r), q.s, f[4 * b + 3]);
+    Io::round_trip(h);
+    f[4 * b + 0] = fmaf(-(s2 * p.r), p.c, h[0]);
+    f[4 * b + 1] = fmaf(-(s2 * p.r), p.s, h[1]);
+    f[4 * b + 2] = fmaf(-(s2 * q.r), q.c, h[2]);
+    f[4 * b + 3] = fmaf(-(s2 * q.r), q.s, h[3]);
+  }
+}
 
 // Segment of `tile`; `seg` is the CTA's cursor and only moves forward.
 __device__ __forceinline__ const SegDesc* find_segment(const SegDesc* __restrict__ segs,
@@ -86,17 +162,73 @@ __device__ __forceinline__ const SegDesc* find_segment(const SegDesc* __restrict
   return segs + seg;
 }
 
+// Whether every global index of the tile's elements [t0, t0 + tile) (clipped
+// to the segment) shares the high word of its Philox block counter, i.e. the
+// tile does not cross a multiple of 2^34 in index space.
+__device__ __forceinline__ bool uniform_hi(uint64_t index_base, uint64_t t0, uint64_t tile,
+                                           uint64_t numel) {
+  const uint64_t last = index_base + (t0 + tile < numel ? t0 + tile : numel) - 1;
+  return ((index_base + t0) >> 34) == (last >> 34);
+}
+
+// One tile of the perturb/restore pass (kTwo: fused restore + perturb; kSame:
+// both steps use one seed, whose noise is generated once).
+template <class Io, bool kTwo, bool kSame, bool kUniformHi>
+__device__ __forceinline__ void axpy_tile(typename Io::Scalar* base, uint64_t numel,
+                                          uint64_t index_base, uint64_t t0, PhiloxKey key,
+                                          float scale, PhiloxKey key2, float scale2) {
+  constexpr int V = Io::kVec;
+  const uint32_t j_hi = static_cast<uint32_t>((index_base + t0) >> 34);
+  const auto gen = make_gen<kUniformHi>(key, j_hi);
+  const auto gen2 = make_gen<kUniformHi && kTwo && !kSame>(key2, j_hi);
+  uint4 v[kVecsPerThread];
+#pragma unroll
+  for (int u = 0; u < kVecsPerThread; ++u) {
+    const uint64_t e = t0 + static_cast<uint64_t>(u * kBlockThreads + threadIdx.x) * V;
+    if (e + V <= numel) v[u] = *reinterpret_cast<const uint4*>(base + e);
+  }
+#pragma unroll
+  for (int u = 0; u < kVecsPerThread; ++u) {
+    const uint64_t e = t0 + static_cast<uint64_t>(u * kBlockThreads + threadIdx.x) * V;
+    if (e >= numel) continue;
+    const bool full = e + V <= numel;
+    const int rem = full ? V : static_cast<int>(numel - e);
+    float f[V];
+    if (full) {
+      Io::unpack(v[u], f);
+    } else {  // ragged end of a segment
+#pragma unroll
+      for (int k = 0; k < V; ++k) f[k] = k < rem ? Io::to_f32(base[e + k]) : 0.0f;
+    }
+    if (kSame) {
+      add_scaled_noise_twice<Io, V>(gen, index_base + e, scale, scale2, f);
+    } else {
+      add_scaled_noise<V>(gen, index_base + e, scale, f);
+      if (kTwo) {
+        Io::round_trip(f);
+        add_scaled_noise<V>(gen2, index_base + e, scale2, f);
+      }
+    }
+    if (full) {
+      *reinterpret_cast<uint4*>(base + e) = Io::pack(f);
+    } else {
+#pragma unroll
+      for (int k = 0; k < V; ++k)
+        if (k < rem) base[e + k] = Io::from_f32(f[k]);
+    }
+  }
+}
+
 // theta[g] <- round(theta[g] + scale * eps_seed[g]) over every segment; with
 // kTwo, a second step round(. + scale2 * eps_seed2[g]) follows in registers,
 // after the first result has been rounded to the storage type exactly as a
 // separate launch would store it (restore of one member fused with the
 // perturb of the next).
-template <class Io, bool kTwo>
-__global__ void __launch_bounds__(kBlockThreads)
+template <class Io, bool kTwo, bool kSame>
+__global__ void ES_AXPY_BOUNDS
 axpy_noise_kernel(const SegDesc* __restrict__ segs, uint64_t total_tiles, PhiloxKey key,
                   float scale, PhiloxKey key2, float scale2) {
-  constexpr int V = Io::kVec;
-  constexpr uint64_t kTile = static_cast<uint64_t>(kBlockThreads) * kVecsPerThread * V;
+  constexpr uint64_t kTile = static_cast<uint64_t>(kBlockThreads) * kVecsPerThread * Io::kVec;
   using S = typename Io::Scalar;
   int seg = 0;
   for (uint64_t tile = blockIdx.x; tile < total_tiles; tile += gridDim.x) {
@@ -105,66 +237,151 @@ axpy_noise_kernel(const SegDesc* __restrict__ segs, uint64_t total_tiles, Philox
     const uint64_t numel = d->numel;
     const uint64_t index_base = d->index_base;
     const uint64_t t0 = (tile - d->tile_begin) * kTile;
+    if (uniform_hi(index_base, t0, kTile, numel))
+      axpy_tile<Io, kTwo, kSame, true>(base, numel, index_base, t0, key, scale, key2, scale2);
+    else
+      axpy_tile<Io, kTwo, kSame, false>(base, numel, index_base, t0, key, scale, key2, scale2);
+  }
+}
 
-    uint4 v[kVecsPerThread];
+// One tile of a single-generation update without a trailing perturb
+// (es_update): acc = sum_i c_i eps_i (fp32, ascending i), then theta + acc
+// rounded once; theta read and written once.
+template <class Io, bool kUniformHi>
+__device__ __forceinline__ void update_tile_single(typename Io::Scalar* base, uint64_t numel,
+                                                   uint64_t index_base, uint64_t t0, int n,
+                                                   const PhiloxKey* s_key, const float* s_coeff) {
+  constexpr int V = Io::kVec;
+  const uint32_t j_hi = static_cast<uint32_t>((index_base + t0) >> 34);
+  uint4 v[kVecsPerThread];
 #pragma unroll
-    for (int u = 0; u < kVecsPerThread; ++u) {
-      const uint64_t e = t0 + static_cast<uint64_t>(u * kBlockThreads + threadIdx.x) * V;
-      if (e + V <= numel) v[u] = *reinterpret_cast<const uint4*>(base + e);
-    }
+  for (int u = 0; u < kVecsPerThread; ++u) {
+    const uint64_t e = t0 + static_cast<uint64_t>(u * kBlockThreads + threadIdx.x) * V;
+    if (e + V <= numel) v[u] = *reinterpret_cast<const uint4*>(base + e);
+  }
+  float acc[kVecsPerThread][V];
+#pragma unroll
+  for (int u = 0; u < kVecsPerThread; ++u)
+#pragma unroll
+    for (int k = 0; k < V; ++k) acc[u][k] = 0.0f;
+#pragma unroll 1
+  for (int i = 0; i < n; ++i) {
+    const auto gen = make_gen<kUniformHi>(s_key[i], j_hi);
+    const float c = s_coeff[i];
 #pragma unroll
     for (int u = 0; u < kVecsPerThread; ++u) {
       const uint64_t e = t0 + static_cast<uint64_t>(u * kBlockThreads + threadIdx.x) * V;
       if (e >= numel) continue;
-      float eps[V];
-      Io::noise(index_base + e, key, eps);
-      if (e + V <= numel) {
-        float f[V];
-        Io::unpack(v[u], f);
+      add_scaled_noise<V>(gen, index_base + e, c, acc[u]);
+    }
+  }
 #pragma unroll
-        for (int k = 0; k < V; ++k) f[k] = fmaf(scale, eps[k], f[k]);
-        if (kTwo) {
-          Io::round_trip(f);
-          Io::noise(index_base + e, key2, eps);
+  for (int u = 0; u < kVecsPerThread; ++u) {
+    const uint64_t e = t0 + static_cast<uint64_t>(u * kBlockThreads + threadIdx.x) * V;
+    if (e >= numel) continue;
+    if (e + V <= numel) {
+      float f[V];
+      Io::unpack(v[u], f);
 #pragma unroll
-          for (int k = 0; k < V; ++k) f[k] = fmaf(scale2, eps[k], f[k]);
-        }
-        *reinterpret_cast<uint4*>(base + e) = Io::pack(f);
-      } else {  // ragged end of a segment
-        const int rem = static_cast<int>(numel - e);
-        float f[V];
+      for (int k = 0; k < V; ++k) f[k] = f[k] + acc[u][k];
+      *reinterpret_cast<uint4*>(base + e) = Io::pack(f);
+    } else {
+      const int rem = static_cast<int>(numel - e);
 #pragma unroll
-        for (int k = 0; k < V; ++k)
-          f[k] = k < rem ? fmaf(scale, eps[k], Io::to_f32(base[e + k])) : 0.0f;
-        if (kTwo) {
-          Io::noise(index_base + e, key2, eps);
-#pragma unroll
-          for (int k = 0; k < V; ++k) f[k] = fmaf(scale2, eps[k], Io::round_trip1(f[k]));
-        }
-#pragma unroll
-        for (int k = 0; k < V; ++k)
-          if (k < rem) base[e + k] = Io::from_f32(f[k]);
-      }
+      for (int k = 0; k < V; ++k)
+        if (k < rem) base[e + k] = Io::from_f32(Io::to_f32(base[e + k]) + acc[u][k]);
     }
   }
 }
 
-// theta[g] <- round(theta[g] + sum_i c_i eps_{s_i}[g]): fp32 accumulation in
-// ascending i, one rounding; theta read and written once.
-template <class Io>
-__global__ void __launch_bounds__(kBlockThreads)
+// One tile of a fused update launch. Theta stays in registers in storage
+// form; generation g adds acc_g = sum_{i in g} c_i eps_i (fp32, ascending i)
+// and rounds once, exactly as a separate launch per generation would store it;
+// an optional trailing perturb step follows. Theta is read and written once.
+template <class Io, bool kUniformHi>
+__device__ __forceinline__ void update_tile(typename Io::Scalar* base, uint64_t numel,
+                                            uint64_t index_base, uint64_t t0,
+                                            const UpdateArgs& args, const PhiloxKey* s_key,
+                                            const float* s_coeff, const uint16_t* s_gen_end) {
+  constexpr int V = Io::kVec;
+  const uint32_t j_hi = static_cast<uint32_t>((index_base + t0) >> 34);
+  uint4 v[kVecsPerThread];
+#pragma unroll
+  for (int u = 0; u < kVecsPerThread; ++u) {
+    const uint64_t e = t0 + static_cast<uint64_t>(u * kBlockThreads + threadIdx.x) * V;
+    if (e + V <= numel)
+      v[u] = *reinterpret_cast<const uint4*>(base + e);
+    else if (e < numel)
+      v[u] = Io::load_partial(base, e, static_cast<int>(numel - e));
+  }
+  int i = 0;
+#pragma unroll 1
+  for (int g = 0; g < args.n_gen; ++g) {
+    float acc[kVecsPerThread][V];
+#pragma unroll
+    for (int u = 0; u < kVecsPerThread; ++u)
+#pragma unroll
+      for (int k = 0; k < V; ++k) acc[u][k] = 0.0f;
+    const int end = s_gen_end[g];
+#pragma unroll 1
+    for (; i < end; ++i) {
+      const auto gen = make_gen<kUniformHi>(s_key[i], j_hi);
+      const float c = s_coeff[i];
+#pragma unroll
+      for (int u = 0; u < kVecsPerThread; ++u) {
+        const uint64_t e = t0 + static_cast<uint64_t>(u * kBlockThreads + threadIdx.x) * V;
+        if (e >= numel) continue;
+        add_scaled_noise<V>(gen, index_base + e, c, acc[u]);
+      }
+    }
+#pragma unroll
+    for (int u = 0; u < kVecsPerThread; ++u) {
+      float f[V];
+      Io::unpack(v[u], f);
+#pragma unroll
+      for (int k = 0; k < V; ++k) f[k] = f[k] + acc[u][k];
+      v[u] = Io::pack(f);
+    }
+  }
+  if (args.perturb) {
+    const auto gen = make_gen<kUniformHi>(PhiloxKey{args.pkey[0], args.pkey[1]}, j_hi);
+#pragma unroll
+    for (int u = 0; u < kVecsPerThread; ++u) {
+      const uint64_t e = t0 + static_cast<uint64_t>(u * kBlockThreads + threadIdx.x) * V;
+      if (e >= numel) continue;
+      float f[V];
+      Io::unpack(v[u], f);
+      add_scaled_noise<V>(gen, index_base + e, args.pscale, f);
+      v[u] = Io::pack(f);
+    }
+  }
+#pragma unroll
+  for (int u = 0; u < kVecsPerThread; ++u) {
+    const uint64_t e = t0 + static_cast<uint64_t>(u * kBlockThreads + threadIdx.x) * V;
+    if (e + V <= numel)
+      *reinterpret_cast<uint4*>(base + e) = v[u];
+    else if (e < numel)
+      Io::store_partial(base, e, static_cast<int>(numel - e), v[u]);
+  }
+}
+
+// Fused update launch (es_update, es_replay, es_update_perturb): for each
+// generation g, theta[g] <- round(theta[g] + sum_{i in g} c_i eps_{s_i}[g]),
+// then optionally theta <- round(theta + pscale * eps_pseed).
+template <class Io, bool kSingle>
+__global__ void ES_UPDATE_BOUNDS
 update_kernel(const SegDesc* __restrict__ segs, uint64_t total_tiles,
               const __grid_constant__ UpdateArgs args) {
-  constexpr int V = Io::kVec;
-  constexpr uint64_t kTile = static_cast<uint64_t>(kBlockThreads) * kVecsPerThread * V;
+  constexpr uint64_t kTile = static_cast<uint64_t>(kBlockThreads) * kVecsPerThread * Io::kVec;
   using S = typename Io::Scalar;
   __shared__ PhiloxKey s_key[ES_MAX_SEEDS];
   __shared__ float s_coeff[ES_MAX_SEEDS];
-  const int n = args.n;
-  for (int i = threadIdx.x; i < n; i += blockDim.x) {
+  __shared__ uint16_t s_gen_end[kMaxGenerations];
+  for (int i = threadIdx.x; i < args.n; i += blockDim.x) {
     s_key[i] = PhiloxKey{args.key[i][0], args.key[i][1]};
     s_coeff[i] = args.coeff[i];
   }
+  for (int g = threadIdx.x; g < args.n_gen; g += blockDim.x) s_gen_end[g] = args.gen_end[g];
   __syncthreads();
 
   int seg = 0;
@@ -174,50 +391,17 @@ update_kernel(const SegDesc* __restrict__ segs, uint64_t total_tiles,
     const uint64_t numel = d->numel;
     const uint64_t index_base = d->index_base;
     const uint64_t t0 = (tile - d->tile_begin) * kTile;
-
-    uint4 v[kVecsPerThread];
-#pragma unroll
-    for (int u = 0; u < kVecsPerThread; ++u) {
-      const uint64_t e = t0 + static_cast<uint64_t>(u * kBlockThreads + threadIdx.x) * V;
-      if (e + V <= numel) v[u] = *reinterpret_cast<const uint4*>(base + e);
-    }
-    float acc[kVecsPerThread][V];
-#pragma unroll
-    for (int u = 0; u < kVecsPerThread; ++u)
-#pragma unroll
-      for (int k = 0; k < V; ++k) acc[u][k] = 0.0f;
-
-#pragma unroll 1
-    for (int i = 0; i < n; ++i) {
-      const PhiloxKey key = s_key[i];
-      const float c = s_coeff[i];
-#pragma unroll
-      for (int u = 0; u < kVecsPerThread; ++u) {
-        const uint64_t e = t0 + static_cast<uint64_t>(u * kBlockThreads + threadIdx.x) * V;
-        if (e >= numel) continue;
-        float eps[V];
-        Io::noise(index_base + e, key, eps);
-#pragma unroll
-        for (int k = 0; k < V; ++k) acc[u][k] = fmaf(c, eps[k], acc[u][k]);
-      }
-    }
-
-#pragma unroll
-    for (int u = 0; u < kVecsPerThread; ++u) {
-      const uint64_t e = t0 + static_cast<uint64_t>(u * kBlockThreads + threadIdx.x) * V;
-      if (e >= numel) continue;
-      if (e + V <= numel) {
-        float f[V];
-        Io::unpack(v[u], f);
-#pragma unroll
-        for (int k = 0; k < V; ++k) f[k] = f[k] + acc[u][k];
-        *reinterpret_cast<uint4*>(base + e) = Io::pack(f);
-      } else {
-        const int rem = static_cast<int>(numel - e);
-#pragma unroll
-        for (int k = 0; k < V; ++k)
-          if (k < rem) base[e + k] = Io::from_f32(Io::to_f32(base[e + k]) + acc[u][k]);
-      }
+    const bool uhi = uniform_hi(index_base, t0, kTile, numel);
+    if constexpr (kSingle) {
+      if (uhi)
+        update_tile_single<Io, true>(base, numel, index_base, t0, args.n, s_key, s_coeff);
+      else
+        update_tile_single<Io, false>(base, numel, index_base, t0, args.n, s_key, s_coeff);
+    } else {
+      if (uhi)
+        update_tile<Io, true>(base, numel, index_base, t0, args, s_key, s_coeff, s_gen_end);
+      else
+        update_tile<Io, false>(base, numel, index_base, t0, args, s_key, s_coeff, s_gen_end);
     }
   }
 }
@@ -242,13 +426,20 @@ noise_fill_kernel(uint64_t index_base, uint64_t n, PhiloxKey key, float* __restr
   }
 }
 
-// out[4t .. 4t+3] = Philox words of block block_base + t.
+// out[4t .. 4t+3] = Philox words of block block_base + t. Even and odd blocks
+// go through the two implementations of the rounds (general, and with the
+// per-tile constants of philox_tile); they give identical words, and this lets
+// a bit-exact check of this output cover both.
 __global__ void __launch_bounds__(kBlockThreads)
 noise_bits_kernel(uint64_t block_base, uint64_t nblocks, PhiloxKey key, uint4* __restrict__ out) {
   const uint64_t stride = static_cast<uint64_t>(gridDim.x) * blockDim.x;
   for (uint64_t t = static_cast<uint64_t>(blockIdx.x) * blockDim.x + threadIdx.x; t < nblocks;
-       t += stride)
-    out[t] = philox_block(block_base + t, key);
+       t += stride) {
+    const uint64_t j = block_base + t;
+    out[t] = (j & 1) ? philox_block_tile(static_cast<uint32_t>(j),
+                                         philox_tile(static_cast<uint32_t>(j >> 32), key))
+                     : philox_block(j, key);
+  }
 }
 
 // out[2k], out[2k+1] = Box-Muller pair of words[2k], words[2k+1].
@@ -277,15 +468,15 @@ int persistent_grid(K kernel, uint64_t work_items) {
   return grid < 1 ? 1 : static_cast<int>(grid);
 }
 
-template <bool kTwo>
+template <bool kTwo, bool kSame>
 cudaError_t launch_axpy(const PlanView& plan, PhiloxKey key, float scale, PhiloxKey key2,
                         float scale2, cudaStream_t stream) {
   if (plan.dtype == ES_BF16) {
-    auto k = axpy_noise_kernel<Bf16Io, kTwo>;
+    auto k = axpy_noise_kernel<Bf16Io, kTwo, kSame>;
     k<<<persistent_grid(k, plan.total_tiles), kBlockThreads, 0, stream>>>(
         plan.segs, plan.total_tiles, key, scale, key2, scale2);
   } else {
-    auto k = axpy_noise_kernel<F32Io, kTwo>;
+    auto k = axpy_noise_kernel<F32Io, kTwo, kSame>;
     k<<<persistent_grid(k, plan.total_tiles), kBlockThreads, 0, stream>>>(
         plan.segs, plan.total_tiles, key, scale, key2, scale2);
   }
@@ -296,21 +487,27 @@ cudaError_t launch_axpy(const PlanView& plan, PhiloxKey key, float scale, Philox
 
 cudaError_t launch_axpy_noise(const PlanView& plan, uint64_t seed, float scale,
                               cudaStream_t stream) {
-  return launch_axpy<false>(plan, philox_key(seed), scale, PhiloxKey{0u, 0u}, 0.0f, stream);
+  return launch_axpy<false, false>(plan, philox_key(seed), scale, PhiloxKey{0u, 0u}, 0.0f,
+                                   stream);
 }
 
 cudaError_t launch_axpy_noise2(const PlanView& plan, uint64_t seed, float scale, uint64_t seed2,
                                float scale2, cudaStream_t stream) {
-  return launch_axpy<true>(plan, philox_key(seed), scale, philox_key(seed2), scale2, stream);
+  if (seed == seed2)
+    return launch_axpy<true, true>(plan, philox_key(seed), scale, philox_key(seed2), scale2,
+                                   stream);
+  return launch_axpy<true, false>(plan, philox_key(seed), scale, philox_key(seed2), scale2,
+                                  stream);
 }
 
 cudaError_t launch_update(const PlanView& plan, const UpdateArgs& args, cudaStream_t stream) {
+  const bool single = args.n_gen == 1 && !args.perturb;
   if (plan.dtype == ES_BF16) {
-    auto k = update_kernel<Bf16Io>;
+    auto k = single ? update_kernel<Bf16Io, true> : update_kernel<Bf16Io, false>;
     k<<<persistent_grid(k, plan.total_tiles), kBlockThreads, 0, stream>>>(
         plan.segs, plan.total_tiles, args);
   } else {
-    auto k = update_kernel<F32Io>;
+    auto k = single ? update_kernel<F32Io, true> : update_kernel<F32Io, false>;
     k<<<persistent_grid(k, plan.total_tiles), kBlockThreads, 0, stream>>>(
         plan.segs, plan.total_tiles, args);
   }

@@ -55,6 +55,54 @@ __device__ __forceinline__ uint4 philox_block(uint64_t j, PhiloxKey key) {
   return make_uint4(c0, c1, c2, c3);
 }
 
+// The same ten rounds for the blocks of one tile that share the high counter
+// word j_hi. With counter (j_lo, j_hi, 0, 0) the first round's second product
+// is zero and its word 0 is j_hi ^ k0, so the second round's first product
+// depends only on (key, j_hi): those parts are computed once per tile
+// (philox_tile) instead of once per block, saving one multiply per block.
+// Bit-identical to philox_block.
+struct PhiloxTile {
+  PhiloxKey key;
+  uint32_t w0;     // word 0 after round 1: j_hi ^ k0
+  uint32_t x2;     // high word of kPhiloxMulA * w0, xored with round 2's k1
+  uint32_t lo2;    // low word of kPhiloxMulA * w0
+};
+
+__device__ __forceinline__ PhiloxTile philox_tile(uint32_t j_hi, PhiloxKey key) {
+  const uint32_t w0 = j_hi ^ key.k0;
+  const uint64_t p = static_cast<uint64_t>(kPhiloxMulA) * w0;
+  return PhiloxTile{key, w0, static_cast<uint32_t>(p >> 32) ^ (key.k1 + kPhiloxWeylB),
+                    static_cast<uint32_t>(p)};
+}
+
+__device__ __forceinline__ uint4 philox_block_tile(uint32_t j_lo, const PhiloxTile& t) {
+  // round 1 (keys k0, k1): products kPhiloxMulA * j_lo and kPhiloxMulB * 0
+  const uint64_t p1 = static_cast<uint64_t>(kPhiloxMulA) * j_lo;
+  const uint32_t a2 = static_cast<uint32_t>(p1 >> 32) ^ t.key.k1;   // word 2
+  const uint32_t a3 = static_cast<uint32_t>(p1);                    // word 3
+  // round 2 (keys k0 + W_A, k1 + W_B): word 0 is t.w0, its product is per tile
+  const uint64_t p2 = static_cast<uint64_t>(kPhiloxMulB) * a2;
+  uint32_t c0 = static_cast<uint32_t>(p2 >> 32) ^ (t.key.k0 + kPhiloxWeylA);  // word 1 was 0
+  uint32_t c1 = static_cast<uint32_t>(p2);
+  uint32_t c2 = t.x2 ^ a3;
+  uint32_t c3 = t.lo2;
+  uint32_t k0 = t.key.k0 + 2u * kPhiloxWeylA, k1 = t.key.k1 + 2u * kPhiloxWeylB;
+#pragma unroll
+  for (int round = 2; round < 10; ++round) {
+    const uint64_t pa = static_cast<uint64_t>(kPhiloxMulA) * c0;
+    const uint64_t pb = static_cast<uint64_t>(kPhiloxMulB) * c2;
+    const uint32_t n0 = static_cast<uint32_t>(pb >> 32) ^ c1 ^ k0;
+    const uint32_t n2 = static_cast<uint32_t>(pa >> 32) ^ c3 ^ k1;
+    c1 = static_cast<uint32_t>(pb);
+    c3 = static_cast<uint32_t>(pa);
+    c0 = n0;
+    c2 = n2;
+    k0 += kPhiloxWeylA;
+    k1 += kPhiloxWeylB;
+  }
+  return make_uint4(c0, c1, c2, c3);
+}
+
 // u = (2m + 1) / 2^24 with m = x >> 9, computed exactly: the bit pattern
 // 0x3F800000 | m is 1 + m 2^-23, and subtracting 1 - 2^-24 (0x3F7FFFFF) leaves
 // (2m + 1) 2^-24, which has at most 24 significant bits.
@@ -64,10 +112,12 @@ __device__ __forceinline__ float uniform_open(uint32_t x) {
 
 // Below this u the radius comes from the hardware log2; above it (u within
 // 2^-10 of 1, where an absolute log2 error would be a large relative error of
-// the small radius) from the series of ln(1 - t), t = 1 - u exact.
+// the small radius) from the series of -ln(1 - t), t = 1 - u exact.
 constexpr float kNearOne = 0.9990234375f;  // 1 - 2^-10
 constexpr float kMinusTwoLn2 = -1.38629436111989061883f;
 constexpr float kTwoPi = 6.28318530717958647692f;
+// -3 pi + 2 pi 2^-24 rounded to float: 2 pi (f - 3/2 + 2^-24) = fma(f, 2 pi, this)
+constexpr float kAngleOffset = -9.42477798f;
 
 __device__ __forceinline__ float sqrt_approx(float x) {
   float r;
@@ -77,37 +127,50 @@ __device__ __forceinline__ float sqrt_approx(float x) {
 
 // radius^2 = -2 ln u for u = uniform_open(x), fast path:
 //   for u <= 1 - 2^-10: -2 ln 2 * log2(u) with the MUFU log2 (__log2f);
-//   for u >  1 - 2^-10: 2t + t^2 + (2/3) t^3 with t = 1 - u (exact), whose
-//     truncation error is below t^3/4 relative (an absolute log2 error there
-//     would be a large relative error of the small radius).
+//   for u >  1 - 2^-10: 2t + t^2 with t = 1 - u (exact); the dropped terms
+//     (2/3 t^3 + ...) are below t^2/3 <= 3.2e-7 relative.
 // Both are evaluated and one is selected, which keeps the code free of
 // divergent branches.
 __device__ __forceinline__ float radius_sq(float u) {
   const float t = 1.0f - u;
-  const float series = t * fmaf(t, fmaf(t, 2.0f / 3.0f, 1.0f), 2.0f);
+  const float series = fmaf(t, t, t + t);
   const float logged = __log2f(u) * kMinusTwoLn2;
   return u > kNearOne ? series : logged;
 }
 
-// One Box-Muller pair, fast path:
-//   radius = sqrt.approx(radius_sq(u_a));
-//   angle: 2 pi u_b = 2 pi s + pi with s = u_b - 1/2 formed exactly from the
-//     bits, so cos/sin of 2 pi u_b are -cos/-sin of 2 pi s, an argument in
-//     (-pi, pi) where __sincosf is accurate.
-// The result is checked against the exact pair over the whole input domain
-// (every 23-bit radius input and every 23-bit angle input) by the test suite;
-// the error stays below 1e-5 * max(1, |eps|).
-__device__ __forceinline__ float2 box_muller(uint32_t xa, uint32_t xb) {
-  const float r = sqrt_approx(radius_sq(uniform_open(xa)));
-  const float s = (__uint_as_float(0x3F800000u | (xb >> 9)) - 1.5f) + 0x1p-24f;
-  float sn, cs;
-  __sincosf(s * kTwoPi, &sn, &cs);
-  return make_float2(-r * cs, -r * sn);
+// Polar form of one Box-Muller pair: eps_even = -r * c, eps_odd = -r * s.
+//   r = sqrt.approx(radius_sq(u_a));
+//   angle: with f = 1 + m_b 2^-23 (bits 0x3F800000 | m_b), 2 pi u_b =
+//     2 pi (f - 3/2 + 2^-24) + pi, so cos/sin of 2 pi u_b are -c/-s with
+//     (s, c) = __sincosf(fma(f, 2 pi, kAngleOffset)), an argument in (-pi, pi)
+//     where __sincosf is accurate; the fma rounds once (|error| < 1e-6).
+// Kernels that add scale * eps fold the scale into r: theta + scale * eps_even
+// = fma(-(scale * r), c, theta).
+// Checked against the exact pair over the whole input domain (every 23-bit
+// radius input and every 23-bit angle input) by the test suite; the error
+// stays below 1e-5 * max(1, |eps|).
+struct Polar {
+  float r, c, s;
+};
+
+__device__ __forceinline__ Polar polar(uint32_t xa, uint32_t xb) {
+  Polar p;
+  p.r = sqrt_approx(radius_sq(uniform_open(xa)));
+  const float f = __uint_as_float(0x3F800000u | (xb >> 9));
+  __sincosf(fmaf(f, kTwoPi, kAngleOffset), &p.s, &p.c);
+  return p;
 }
 
-// eps[4j .. 4j+3] for one seed.
+// One Box-Muller pair, materialised.
+__device__ __forceinline__ float2 box_muller(uint32_t xa, uint32_t xb) {
+  const Polar p = polar(xa, xb);
+  return make_float2(-p.r * p.c, -p.r * p.s);
+}
+
+// eps[4j .. 4j+3] for one seed, materialised.
 __device__ __forceinline__ float4 gaussian4(uint64_t j, PhiloxKey key) {
-  const uint4 x = philox_block(j, key);
+  const uint4 x = philox_block_tile(static_cast<uint32_t>(j),
+                                    philox_tile(static_cast<uint32_t>(j >> 32), key));
   const float2 p = box_muller(x.x, x.y);
   const float2 q = box_muller(x.z, x.w);
   return make_float4(p.x, p.y, q.x, q.y);

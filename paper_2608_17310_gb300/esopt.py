@@ -24,7 +24,7 @@ import numpy as np
 _PKG = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.path.join(_PKG, "_build", "libesopt.so")
 
-ES_MAX_SEEDS = 256
+ES_MAX_SEEDS = 1024
 ES_STATIC_MAX_SEGMENTS = 1024
 
 ES_OK = 0
@@ -82,6 +82,8 @@ def _load() -> ctypes.CDLL:
         "es_restore": (i32, [vp, u64, f32, vp]),
         "es_restore_perturb": (i32, [vp, u64, f32, u64, f32, vp]),
         "es_update": (i32, [vp, P(u64), P(f32), i32, vp]),
+        "es_update_perturb": (i32, [vp, P(u64), P(f32), i32, u64, f32, vp]),
+        "es_replay": (i32, [vp, P(u64), P(f32), P(i32), i32, vp]),
         "es_normalize_rewards": (i32, [P(f64), i32, f64, P(f64)]),
         "es_sigma_cosine": (f64, [f64, f64, i32, i32]),
         "es_update_coeffs": (i32, [P(f64), i32, f64, f64, i32, P(f32)]),
@@ -280,6 +282,30 @@ def es_perturb_noalloc(segments: Sequence[Segment], dtype: int, seed: int, sigma
     arr = _seg_array(segments)
     _check(_load().es_perturb_noalloc(arr, len(segments), dtype, seed, sigma, _stream(stream)),
            "es_perturb_noalloc")
+
+
+def es_update_perturb(plan: Plan, seeds, coeffs, next_seed: int, sigma_next: float,
+                      stream=None) -> None:
+    s = np.ascontiguousarray(seeds, dtype=np.uint64)
+    c = np.ascontiguousarray(coeffs, dtype=np.float32)
+    if s.size != c.size:
+        raise ValueError("seeds and coeffs differ in length")
+    _check(_load().es_update_perturb(plan.handle, s.ctypes.data_as(ctypes.POINTER(ctypes.c_uint64)),
+                                     c.ctypes.data_as(ctypes.POINTER(ctypes.c_float)), s.size,
+                                     next_seed, sigma_next, _stream(stream)), "es_update_perturb")
+
+
+def es_replay(plan: Plan, seeds, coeffs, counts, stream=None) -> None:
+    """Replays generations back to back: counts[g] seeds/coefficients each."""
+    s = np.ascontiguousarray(seeds, dtype=np.uint64)
+    c = np.ascontiguousarray(coeffs, dtype=np.float32)
+    n = np.ascontiguousarray(counts, dtype=np.int32)
+    if s.size != c.size or int(n.sum()) != s.size:
+        raise ValueError("seeds, coeffs and counts do not agree")
+    _check(_load().es_replay(plan.handle, s.ctypes.data_as(ctypes.POINTER(ctypes.c_uint64)),
+                             c.ctypes.data_as(ctypes.POINTER(ctypes.c_float)),
+                             n.ctypes.data_as(ctypes.POINTER(ctypes.c_int)), n.size,
+                             _stream(stream)), "es_replay")
 
 
 # --- host-side generation control ---------------------------------------------------

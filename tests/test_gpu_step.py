@@ -104,18 +104,23 @@ def test_restore_perturb_is_bit_identical_to_the_two_calls(es, oracle, dtype):
     torch.cuda.synchronize()
     mid = [host_values(t) for t in a]
     es.es_restore(plan_a, s1, sig1)
+    torch.cuda.synchronize()
+    restored = [host_values(t) for t in a]
     es.es_perturb(plan_a, s2, sig2)
     es.es_restore_perturb(plan_b, s1, sig1, s2, sig2)
     torch.cuda.synchronize()
     iv = torch.int16 if dtype == "bf16" else torch.int32
     for x, y in zip(a, b):
         assert torch.equal(x.view(iv), y.view(iv))
-    # and against the oracle, step by step
+    # and against the oracle, step by step (each step from the GPU's input)
     g = indices(segs)
     for k in range(len(a)):
-        want = oracle.perturb(oracle.restore(mid[k], g[k], s1, sig1, dtype), g[k], s2, sig2, dtype)
-        tol = noise_abs_tol([oracle.noise_at(s1, g[k]), oracle.noise_at(s2, g[k])], [sig1, sig2])
-        compare(dtype, host_values(b[k]), want, f"restore+perturb seg {k}", tol)
+        tol1 = noise_abs_tol([oracle.noise_at(s1, g[k])], [sig1])
+        compare(dtype, restored[k], oracle.restore(mid[k], g[k], s1, sig1, dtype),
+                f"restore step seg {k}", tol1)
+        tol2 = noise_abs_tol([oracle.noise_at(s2, g[k])], [sig2])
+        compare(dtype, host_values(b[k]), oracle.perturb(restored[k], g[k], s2, sig2, dtype),
+                f"perturb step seg {k}", tol2)
     with pytest.raises(es.EsError) as ei:
         es.es_restore_perturb(plan_b, 1, float("nan"), 2, 1e-3)
     assert ei.value.status == es.ES_ERR_NONFINITE
@@ -124,7 +129,7 @@ def test_restore_perturb_is_bit_identical_to_the_two_calls(es, oracle, dtype):
 
 
 @pytest.mark.parametrize("dtype", ["bf16", "f32"])
-@pytest.mark.parametrize("nseeds", [1, 2, 3, 8, 30, 129, 256])
+@pytest.mark.parametrize("nseeds", [1, 2, 3, 8, 30, 129, 256, 1024])
 def test_update_matches_oracle(es, oracle, dtype, nseeds):
     numels = [9, 8193, 20000, 4096 * 3 + 5]
     tensors = make_params(dtype, numels, seed=2)
@@ -181,7 +186,8 @@ def test_step_argument_errors(es):
         es.es_restore(plan, 1, float("inf"))
     assert ei.value.status == es.ES_ERR_NONFINITE
     with pytest.raises(es.EsError) as ei:
-        es.es_update(plan, np.arange(257, dtype=np.uint64), np.ones(257, np.float32))
+        n = es.ES_MAX_SEEDS + 1
+        es.es_update(plan, np.arange(n, dtype=np.uint64), np.ones(n, np.float32))
     assert ei.value.status == es.ES_ERR_TOO_MANY_SEEDS
     with pytest.raises(es.EsError) as ei:
         es.es_update(plan, [1, 2], np.array([1.0, np.nan], np.float32))
@@ -212,5 +218,111 @@ def test_max_population_update(es, oracle):
     g = indices(segs)[0]
     want = oracle.update(before, g, seeds, coeffs, "f32")
     tol = noise_abs_tol([oracle.noise_at(int(s), g) for s in seeds], coeffs)
-    assert_f32_close(host_values(t), want, "N=256", tol)
+    assert_f32_close(host_values(t), want, f"N={es.ES_MAX_SEEDS}", tol)
+    plan.close()
+
+
+def _int_view(t):
+    return t.view(torch.int16 if t.dtype == torch.bfloat16 else torch.int32)
+
+
+@pytest.mark.parametrize("dtype", ["bf16", "f32"])
+def test_replay_is_bit_identical_to_sequential_updates(es, dtype):
+    numels = [9, 8193, 20000, 4096 * 3 + 5]
+    a = make_params(dtype, numels, seed=8)
+    b = [t.clone() for t in a]
+    bases = [8, 2**34 - 1024, 2**36, 2**50]
+    plan_a, _ = build_plan(es, a, bases)
+    plan_b, _ = build_plan(es, b, bases)
+    rng = np.random.default_rng(9)
+    # 300 generations of 1..8 seeds (over 256 generations and 1024 seeds: several
+    # passes), some all-zero generations and zero coefficients
+    counts = rng.integers(1, 9, size=300)
+    total = int(counts.sum())
+    seeds = rng.integers(0, 2**63, size=total, dtype=np.uint64)
+    coeffs = (1e-3 * rng.standard_normal(total)).astype(np.float32)
+    coeffs[rng.random(total) < 0.1] = 0.0
+    off = 0
+    for g, c in enumerate(counts):
+        if g % 37 == 5:
+            coeffs[off:off + c] = 0.0
+        es.es_update(plan_a, seeds[off:off + c], coeffs[off:off + c])
+        off += c
+    es.es_replay(plan_b, seeds, coeffs, counts)
+    torch.cuda.synchronize()
+    for x, y in zip(a, b):
+        assert torch.equal(_int_view(x), _int_view(y))
+    plan_a.close()
+    plan_b.close()
+
+
+@pytest.mark.parametrize("dtype", ["bf16", "f32"])
+def test_update_perturb_is_bit_identical_to_the_two_calls(es, oracle, dtype):
+    a = make_params(dtype, RAGGED, seed=10)
+    b = [t.clone() for t in a]
+    plan_a, segs = build_plan(es, a, _sparse64(len(RAGGED)))
+    plan_b, _ = build_plan(es, b, _sparse64(len(RAGGED)))
+    before = [host_values(t) for t in a]
+    seeds = np.arange(500, 516, dtype=np.uint64)
+    coeffs = np.linspace(-2e-3, 2e-3, 16).astype(np.float32)
+    es.es_update(plan_a, seeds, coeffs)
+    torch.cuda.synchronize()
+    updated = [host_values(t) for t in a]
+    es.es_perturb(plan_a, 2**40 + 1, 9e-4)
+    es.es_update_perturb(plan_b, seeds, coeffs, 2**40 + 1, 9e-4)
+    torch.cuda.synchronize()
+    for x, y in zip(a, b):
+        assert torch.equal(_int_view(x), _int_view(y))
+    # against the oracle, step by step (each step from the GPU's input)
+    g = indices(segs)
+    for k in (0, 5, 8):
+        tol = noise_abs_tol([oracle.noise_at(int(s), g[k]) for s in seeds], coeffs)
+        compare(dtype, updated[k], oracle.update(before[k], g[k], seeds, coeffs, dtype),
+                f"update step seg {k}", tol)
+        tol = noise_abs_tol([oracle.noise_at(2**40 + 1, g[k])], [9e-4])
+        compare(dtype, host_values(b[k]), oracle.perturb(updated[k], g[k], 2**40 + 1, 9e-4, dtype),
+                f"perturb step seg {k}", tol)
+    # all-zero coefficients: only the perturb
+    es.es_update_perturb(plan_b, seeds, np.zeros(16, np.float32), 77, 1e-3)
+    es.es_perturb(plan_a, 77, 1e-3)
+    torch.cuda.synchronize()
+    for x, y in zip(a, b):
+        assert torch.equal(_int_view(x), _int_view(y))
+    plan_a.close()
+    plan_b.close()
+
+
+@pytest.mark.parametrize("dtype", ["bf16", "f32"])
+def test_antithetic_restore_perturb_reuses_one_seed(es, dtype):
+    # restore (+sigma eps_i) then perturb (-sigma eps_i): the same noise twice
+    a = make_params(dtype, RAGGED, seed=12)
+    b = [t.clone() for t in a]
+    plan_a, _ = build_plan(es, a, _sparse64(len(RAGGED)))
+    plan_b, _ = build_plan(es, b, _sparse64(len(RAGGED)))
+    for p in (plan_a, plan_b):
+        es.es_perturb(p, 31, 5e-2)
+    es.es_restore(plan_a, 31, 5e-2)
+    es.es_perturb(plan_a, 31, -5e-2)
+    es.es_restore_perturb(plan_b, 31, 5e-2, 31, -5e-2)
+    torch.cuda.synchronize()
+    for x, y in zip(a, b):
+        assert torch.equal(_int_view(x), _int_view(y))
+    plan_a.close()
+    plan_b.close()
+
+
+def test_replay_argument_errors(es):
+    t = make_params("bf16", [64], seed=13)[0]
+    plan, _ = build_plan(es, [t])
+    for counts, status in (([0], es.ES_ERR_INVALID_ARG), ([es.ES_MAX_SEEDS + 1], es.ES_ERR_TOO_MANY_SEEDS)):
+        n = sum(counts)
+        with pytest.raises(es.EsError) as ei:
+            es.es_replay(plan, np.arange(n, dtype=np.uint64), np.ones(n, np.float32), counts)
+        assert ei.value.status == status
+    with pytest.raises(es.EsError) as ei:
+        es.es_replay(plan, [1, 2], np.array([1.0, np.inf], np.float32), [2])
+    assert ei.value.status == es.ES_ERR_NONFINITE
+    with pytest.raises(es.EsError) as ei:
+        es.es_update_perturb(plan, [1], [1.0], 2, float("nan"))
+    assert ei.value.status == es.ES_ERR_NONFINITE
     plan.close()
