@@ -169,8 +169,16 @@ def generation_inputs(wl, step: int, n: int):
     return seeds, rewards
 
 
-def run_step(es, plan, wl, step, n, sigma, stream, timers=None, fused=True):
-    """One ES generation through the C ABI. Returns the number of kernels launched."""
+def run_step(es, plan, wl, step, n, sigma, sigma_next, stream, timers=None, fused=True):
+    """One ES generation through the C ABI. Returns the number of kernels launched.
+
+    Fused (the library's steady-state loop): on entry theta carries the
+    perturbation of this generation's first member, applied by the previous
+    step's es_update_perturb; each step does N - 1 es_restore_perturb, one
+    es_restore and one es_update_perturb (update fused with the next
+    generation's first perturb): N perturbs, N restores and one update per
+    generation. Unfused: N x (es_perturb, es_restore), then es_update.
+    """
     seeds, rewards = generation_inputs(wl, step, n)
     launches = [0]
 
@@ -185,7 +193,6 @@ def run_step(es, plan, wl, step, n, sigma, stream, timers=None, fused=True):
     # (the rollout of each perturbed model happens after its perturb; its
     # reward is an input here)
     if fused:
-        call("perturb", es.es_perturb, plan, int(seeds[0]), sigma, stream)
         for i in range(1, n):
             call("restore_perturb", es.es_restore_perturb, plan, int(seeds[i - 1]), sigma,
                  int(seeds[i]), sigma, stream)
@@ -196,11 +203,21 @@ def run_step(es, plan, wl, step, n, sigma, stream, timers=None, fused=True):
             call("restore", es.es_restore, plan, int(seeds[i]), sigma, stream)
     rhat = es.es_normalize_rewards(rewards, 1e-8)
     coeffs = es.es_update_coeffs(rhat, wl.alpha, sigma, es.ES_SCALE_PAPER)
-    if np.any(coeffs != 0):
+    if fused:
+        first_next = int(generation_inputs(wl, step + 1, n)[0][0])
+        call("update_perturb", es.es_update_perturb, plan, seeds, coeffs, first_next,
+             sigma_next, stream)
+    elif np.any(coeffs != 0):
         call("update", es.es_update, plan, seeds, coeffs, stream)
     else:
         es.es_update(plan, seeds, coeffs, stream)   # no launch: the no-update rule
     return launches[0]
+
+
+def start_loop(es, plan, wl, step, n, sigma, stream, fused):
+    """Before the first fused step: perturb with that generation's first member."""
+    if fused:
+        es.es_perturb(plan, int(generation_inputs(wl, step, n)[0][0]), sigma, stream)
 
 
 class KernelTimers:
@@ -241,7 +258,14 @@ GAUSS_PER_ELEM = {"perturb": 1, "restore": 1, "restore_perturb": 2}
 KERNEL_NAME = {"perturb": "axpy_noise_kernel<1 step> (es_perturb)",
                "restore": "axpy_noise_kernel<1 step> (es_restore)",
                "restore_perturb": "axpy_noise_kernel<2 steps> (es_restore_perturb)",
-               "update": "update_kernel (es_update)"}
+               "update": "update_kernel<single generation> (es_update)",
+               "update_perturb": "update_kernel<generations + perturb> (es_update_perturb)"}
+
+
+def gauss_per_elem(kind, n):
+    if kind in GAUSS_PER_ELEM:
+        return GAUSS_PER_ELEM[kind]
+    return n + 1 if kind == "update_perturb" else n
 # Philox4x32-10: 10 rounds x 2 products of 32x32->64 bits per 4 outputs, each
 # product two 32-bit multiplies (high and low word): 10 per Gaussian.
 IMUL_PER_GAUSS = 10
@@ -290,14 +314,15 @@ def run_ours(args, rank, world, dist):
     def sigma_at(t):
         return float(np.float32(es.es_sigma_cosine(sigma0, sigmaT, t, SCHEDULE_T)))
 
+    fused = not args.unfused
+    start_loop(es, plan, wl, 0, n, sigma_at(0), s_handle, fused)
     for w in range(args.warmup):
-        run_step(es, plan, wl, w, n, sigma_at(w), s_handle)
+        run_step(es, plan, wl, w, n, sigma_at(w), sigma_at(w + 1), s_handle, None, fused)
     torch.cuda.synchronize()
     barrier(dist)
     torch.cuda.synchronize()
 
     timers = KernelTimers(torch, stream)
-    fused = not args.unfused
     launches = 0
     ev0 = torch.cuda.Event(enable_timing=True)
     ev1 = torch.cuda.Event(enable_timing=True)
@@ -305,7 +330,8 @@ def run_ours(args, rank, world, dist):
         ev0.record(stream)
         for k in range(args.steps):
             t = args.warmup + k
-            launches += run_step(es, plan, wl, t, n, sigma_at(t), s_handle, timers, fused)
+            launches += run_step(es, plan, wl, t, n, sigma_at(t), sigma_at(t + 1), s_handle,
+                                 timers, fused)
         ev1.record(stream)
         torch.cuda.synchronize()
     barrier(dist)
@@ -323,7 +349,7 @@ def run_ours(args, rank, world, dist):
     kernels = {}
     for name in timers.names():
         mean = timers.mean_ms(name)
-        g = GAUSS_PER_ELEM.get(name, n) * P
+        g = gauss_per_elem(name, n) * P
         gbs = bytes_per_launch / (mean / 1e3) / 1e9
         gps = g / (mean / 1e3)
         hbm_frac, alu_frac = gbs / hbm_gbs, gps / gauss_peak
@@ -347,7 +373,7 @@ def run_ours(args, rank, world, dist):
                                f"{sm_max_mhz:.0f} MHz; {IMUL_PER_GAUSS} multiplies per Gaussian"}
     roof.update({"kernel": d["kernel"], "hbm_frac": d["hbm_frac"], "alu_frac": d["alu_frac"],
                  "algorithmic_bytes_per_launch": bytes_per_launch,
-                 "gaussians_per_launch": GAUSS_PER_ELEM.get(dom, n) * P})
+                 "gaussians_per_launch": gauss_per_elem(dom, n) * P})
 
     e2e = None
     if not args.no_e2e:
@@ -364,7 +390,8 @@ def run_ours(args, rank, world, dist):
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
         "dtype": "f32", "data": "synthetic",
         "config": dict(workload_config(args.workload, n, world), sigma=sigma_at(args.warmup),
-                       generation_loop="fused es_restore_perturb" if fused else "separate calls"),
+                       generation_loop=("es_restore_perturb x (N-1), es_restore, es_update_perturb"
+                                        if fused else "separate calls")),
         "roofline": roof,
         "kernels": kernels,
         "gpu_launches": launches,
@@ -388,7 +415,8 @@ def run_e2e(args, torch, es, plan, params, wl, n, esize, sigma_at, s_handle, dis
     def one(t):
         for h, p in zip(host, params):
             p.copy_(h, non_blocking=True)
-        launches = run_step(es, plan, wl, t, n, sigma_at(t), s_handle, None, fused)
+        launches = run_step(es, plan, wl, t, n, sigma_at(t), sigma_at(t + 1), s_handle, None,
+                            fused)
         for h, p in zip(host, params):
             h.copy_(p, non_blocking=True)
         return launches

@@ -171,22 +171,36 @@ __device__ __forceinline__ bool uniform_hi(uint64_t index_base, uint64_t t0, uin
   return ((index_base + t0) >> 34) == (last >> 34);
 }
 
+// Location of one tile: its segment's storage and the tile's first element.
+template <class Io>
+struct TileRef {
+  typename Io::Scalar* base;
+  uint64_t numel;
+  uint64_t index_base;
+  uint64_t t0;
+};
+
+template <class Io>
+__device__ __forceinline__ TileRef<Io> tile_ref(const SegDesc* __restrict__ segs, int& seg,
+                                                uint64_t tile, uint64_t tile_elems) {
+  const SegDesc* d = find_segment(segs, seg, tile);
+  return TileRef<Io>{static_cast<typename Io::Scalar*>(d->data), d->numel, d->index_base,
+                     (tile - d->tile_begin) * tile_elems};
+}
+
 // One tile of the perturb/restore pass (kTwo: fused restore + perturb; kSame:
-// both steps use one seed, whose noise is generated once).
+// both steps use one seed, whose noise is generated once). v[u] holds the
+// thread's full vectors of the tile.
 template <class Io, bool kTwo, bool kSame, bool kUniformHi>
-__device__ __forceinline__ void axpy_tile(typename Io::Scalar* base, uint64_t numel,
-                                          uint64_t index_base, uint64_t t0, PhiloxKey key,
-                                          float scale, PhiloxKey key2, float scale2) {
+__device__ __forceinline__ void axpy_tile(const TileRef<Io>& r, const uint4 (&v)[kVecsPerThread],
+                                          PhiloxKey key, float scale, PhiloxKey key2,
+                                          float scale2) {
   constexpr int V = Io::kVec;
+  typename Io::Scalar* const base = r.base;
+  const uint64_t numel = r.numel, index_base = r.index_base, t0 = r.t0;
   const uint32_t j_hi = static_cast<uint32_t>((index_base + t0) >> 34);
   const auto gen = make_gen<kUniformHi>(key, j_hi);
   const auto gen2 = make_gen<kUniformHi && kTwo && !kSame>(key2, j_hi);
-  uint4 v[kVecsPerThread];
-#pragma unroll
-  for (int u = 0; u < kVecsPerThread; ++u) {
-    const uint64_t e = t0 + static_cast<uint64_t>(u * kBlockThreads + threadIdx.x) * V;
-    if (e + V <= numel) v[u] = *reinterpret_cast<const uint4*>(base + e);
-  }
 #pragma unroll
   for (int u = 0; u < kVecsPerThread; ++u) {
     const uint64_t e = t0 + static_cast<uint64_t>(u * kBlockThreads + threadIdx.x) * V;
@@ -219,6 +233,16 @@ __device__ __forceinline__ void axpy_tile(typename Io::Scalar* base, uint64_t nu
   }
 }
 
+template <class Io, bool kTwo, bool kSame>
+__device__ __forceinline__ void axpy_dispatch(const TileRef<Io>& r, const uint4 (&v)[kVecsPerThread],
+                                              uint64_t tile_elems, PhiloxKey key, float scale,
+                                              PhiloxKey key2, float scale2) {
+  if (uniform_hi(r.index_base, r.t0, tile_elems, r.numel))
+    axpy_tile<Io, kTwo, kSame, true>(r, v, key, scale, key2, scale2);
+  else
+    axpy_tile<Io, kTwo, kSame, false>(r, v, key, scale, key2, scale2);
+}
+
 // theta[g] <- round(theta[g] + scale * eps_seed[g]) over every segment; with
 // kTwo, a second step round(. + scale2 * eps_seed2[g]) follows in registers,
 // after the first result has been rounded to the storage type exactly as a
@@ -228,31 +252,33 @@ template <class Io, bool kTwo, bool kSame>
 __global__ void ES_AXPY_BOUNDS
 axpy_noise_kernel(const SegDesc* __restrict__ segs, uint64_t total_tiles, PhiloxKey key,
                   float scale, PhiloxKey key2, float scale2) {
-  constexpr uint64_t kTile = static_cast<uint64_t>(kBlockThreads) * kVecsPerThread * Io::kVec;
-  using S = typename Io::Scalar;
+  constexpr int V = Io::kVec;
+  constexpr uint64_t kTile = static_cast<uint64_t>(kBlockThreads) * kVecsPerThread * V;
   int seg = 0;
   for (uint64_t tile = blockIdx.x; tile < total_tiles; tile += gridDim.x) {
-    const SegDesc* d = find_segment(segs, seg, tile);
-    S* const base = static_cast<S*>(d->data);
-    const uint64_t numel = d->numel;
-    const uint64_t index_base = d->index_base;
-    const uint64_t t0 = (tile - d->tile_begin) * kTile;
-    if (uniform_hi(index_base, t0, kTile, numel))
-      axpy_tile<Io, kTwo, kSame, true>(base, numel, index_base, t0, key, scale, key2, scale2);
-    else
-      axpy_tile<Io, kTwo, kSame, false>(base, numel, index_base, t0, key, scale, key2, scale2);
+    const TileRef<Io> cur = tile_ref<Io>(segs, seg, tile, kTile);
+    uint4 v[kVecsPerThread];
+#pragma unroll
+    for (int u = 0; u < kVecsPerThread; ++u) {
+      const uint64_t e = cur.t0 + static_cast<uint64_t>(u * kBlockThreads + threadIdx.x) * V;
+      if (e + V <= cur.numel) v[u] = *reinterpret_cast<const uint4*>(cur.base + e);
+    }
+    axpy_dispatch<Io, kTwo, kSame>(cur, v, kTile, key, scale, key2, scale2);
   }
 }
 
-// One tile of a single-generation update without a trailing perturb
-// (es_update): acc = sum_i c_i eps_i (fp32, ascending i), then theta + acc
-// rounded once; theta read and written once.
-template <class Io, bool kUniformHi>
+// One tile of a single-generation update (es_update; with kPerturb also the
+// trailing perturb of es_update_perturb): acc = sum_i c_i eps_i (fp32,
+// ascending i), then theta + acc rounded once (then + pscale * eps_pseed,
+// rounded again); theta read and written once.
+template <class Io, bool kUniformHi, bool kPerturb>
 __device__ __forceinline__ void update_tile_single(typename Io::Scalar* base, uint64_t numel,
-                                                   uint64_t index_base, uint64_t t0, int n,
-                                                   const PhiloxKey* s_key, const float* s_coeff) {
+                                                   uint64_t index_base, uint64_t t0,
+                                                   const UpdateArgs& args, const PhiloxKey* s_key,
+                                                   const float* s_coeff) {
   constexpr int V = Io::kVec;
   const uint32_t j_hi = static_cast<uint32_t>((index_base + t0) >> 34);
+  const int n = args.n;
   uint4 v[kVecsPerThread];
 #pragma unroll
   for (int u = 0; u < kVecsPerThread; ++u) {
@@ -275,21 +301,32 @@ __device__ __forceinline__ void update_tile_single(typename Io::Scalar* base, ui
       add_scaled_noise<V>(gen, index_base + e, c, acc[u]);
     }
   }
+  const auto pgen = make_gen<kUniformHi && kPerturb>(PhiloxKey{args.pkey[0], args.pkey[1]}, j_hi);
 #pragma unroll
   for (int u = 0; u < kVecsPerThread; ++u) {
     const uint64_t e = t0 + static_cast<uint64_t>(u * kBlockThreads + threadIdx.x) * V;
     if (e >= numel) continue;
-    if (e + V <= numel) {
-      float f[V];
+    const bool full = e + V <= numel;
+    const int rem = full ? V : static_cast<int>(numel - e);
+    float f[V];
+    if (full) {
       Io::unpack(v[u], f);
+    } else {
 #pragma unroll
-      for (int k = 0; k < V; ++k) f[k] = f[k] + acc[u][k];
+      for (int k = 0; k < V; ++k) f[k] = k < rem ? Io::to_f32(base[e + k]) : 0.0f;
+    }
+#pragma unroll
+    for (int k = 0; k < V; ++k) f[k] = f[k] + acc[u][k];
+    if (kPerturb) {
+      Io::round_trip(f);
+      add_scaled_noise<V>(pgen, index_base + e, args.pscale, f);
+    }
+    if (full) {
       *reinterpret_cast<uint4*>(base + e) = Io::pack(f);
     } else {
-      const int rem = static_cast<int>(numel - e);
 #pragma unroll
       for (int k = 0; k < V; ++k)
-        if (k < rem) base[e + k] = Io::from_f32(Io::to_f32(base[e + k]) + acc[u][k]);
+        if (k < rem) base[e + k] = Io::from_f32(f[k]);
     }
   }
 }
@@ -368,7 +405,9 @@ __device__ __forceinline__ void update_tile(typename Io::Scalar* base, uint64_t 
 // Fused update launch (es_update, es_replay, es_update_perturb): for each
 // generation g, theta[g] <- round(theta[g] + sum_{i in g} c_i eps_{s_i}[g]),
 // then optionally theta <- round(theta + pscale * eps_pseed).
-template <class Io, bool kSingle>
+// kSingle: one generation (update_tile_single, with a trailing perturb when
+// kPerturb); otherwise the general form (update_tile).
+template <class Io, bool kSingle, bool kPerturb>
 __global__ void ES_UPDATE_BOUNDS
 update_kernel(const SegDesc* __restrict__ segs, uint64_t total_tiles,
               const __grid_constant__ UpdateArgs args) {
@@ -394,9 +433,9 @@ update_kernel(const SegDesc* __restrict__ segs, uint64_t total_tiles,
     const bool uhi = uniform_hi(index_base, t0, kTile, numel);
     if constexpr (kSingle) {
       if (uhi)
-        update_tile_single<Io, true>(base, numel, index_base, t0, args.n, s_key, s_coeff);
+        update_tile_single<Io, true, kPerturb>(base, numel, index_base, t0, args, s_key, s_coeff);
       else
-        update_tile_single<Io, false>(base, numel, index_base, t0, args.n, s_key, s_coeff);
+        update_tile_single<Io, false, kPerturb>(base, numel, index_base, t0, args, s_key, s_coeff);
     } else {
       if (uhi)
         update_tile<Io, true>(base, numel, index_base, t0, args, s_key, s_coeff, s_gen_end);
@@ -500,18 +539,18 @@ cudaError_t launch_axpy_noise2(const PlanView& plan, uint64_t seed, float scale,
                                   stream);
 }
 
-cudaError_t launch_update(const PlanView& plan, const UpdateArgs& args, cudaStream_t stream) {
-  const bool single = args.n_gen == 1 && !args.perturb;
-  if (plan.dtype == ES_BF16) {
-    auto k = single ? update_kernel<Bf16Io, true> : update_kernel<Bf16Io, false>;
-    k<<<persistent_grid(k, plan.total_tiles), kBlockThreads, 0, stream>>>(
-        plan.segs, plan.total_tiles, args);
-  } else {
-    auto k = single ? update_kernel<F32Io, true> : update_kernel<F32Io, false>;
-    k<<<persistent_grid(k, plan.total_tiles), kBlockThreads, 0, stream>>>(
-        plan.segs, plan.total_tiles, args);
-  }
+template <class Io>
+cudaError_t launch_update_io(const PlanView& plan, const UpdateArgs& args, cudaStream_t stream) {
+  auto k = update_kernel<Io, false, false>;
+  if (args.n_gen == 1) k = args.perturb ? update_kernel<Io, true, true> : update_kernel<Io, true, false>;
+  k<<<persistent_grid(k, plan.total_tiles), kBlockThreads, 0, stream>>>(plan.segs, plan.total_tiles,
+                                                                          args);
   return cudaGetLastError();
+}
+
+cudaError_t launch_update(const PlanView& plan, const UpdateArgs& args, cudaStream_t stream) {
+  return plan.dtype == ES_BF16 ? launch_update_io<Bf16Io>(plan, args, stream)
+                               : launch_update_io<F32Io>(plan, args, stream);
 }
 
 cudaError_t launch_noise_bits(uint64_t seed, uint64_t block_base, uint64_t nblocks,
