@@ -304,7 +304,7 @@ def run_ours(args, rank, world, dist):
     specs = I.shapes_for(args.workload)
     dtype = torch.bfloat16 if wl.dtype == "bf16" else torch.float32
     esize = 2 if wl.dtype == "bf16" else 4
-    params = I.init_params_torch(specs, dtype, "cuda", seed=0)
+    flat, params = I.init_params_flat(specs, dtype, "cuda", seed=0)
     plan = es.plan_from_tensors(params)
     P = plan.numel
     stream = torch.cuda.current_stream()
@@ -377,8 +377,8 @@ def run_ours(args, rank, world, dist):
 
     e2e = None
     if not args.no_e2e:
-        e2e = run_e2e(args, torch, es, plan, params, wl, n, esize, sigma_at, s_handle, dist, world,
-                      fused)
+        e2e = run_e2e(args, torch, es, plan, flat, params, wl, n, esize, sigma_at, s_handle, dist,
+                      world, fused)
 
     cpu = None
     if not args.no_cpu_baseline and rank == 0 and world == 1:
@@ -404,39 +404,102 @@ def run_ours(args, rank, world, dist):
         print(json.dumps(out), flush=True)
 
 
-def run_e2e(args, torch, es, plan, params, wl, n, esize, sigma_at, s_handle, dist, world, fused):
-    """Same step with the parameters in pinned host memory: H2D copy, step, D2H copy."""
-    host = [torch.empty(p.shape, dtype=p.dtype, pin_memory=True) for p in params]
-    for h, p in zip(host, params):
-        h.copy_(p)
+def run_e2e(args, torch, es, plan, flat, params, wl, n, esize, sigma_at, s_handle, dist, world,
+            fused, groups=8, nstreams=4):
+    """Same generation with the parameter set in pinned host memory: every step
+    copies it to the device, runs the generation through the C ABI and copies it
+    back. The tensors are split into `groups` contiguous groups with a plan
+    each, so that each group's first pass starts when its copy has landed and
+    its copy back starts when its last pass is done (the middle passes use the
+    whole plan). The results are those of the unsplit calls: every call is
+    elementwise."""
+    host = torch.empty(flat.shape, dtype=flat.dtype, pin_memory=True)
+    host.copy_(flat)
     stream = torch.cuda.current_stream()
-    bytes_per_copy = sum(p.numel() for p in params) * esize
+    copy_streams = [torch.cuda.Stream() for _ in range(nstreams)]
+    bytes_per_copy = flat.numel() * esize
+    # contiguous groups of tensors with about equal bytes
+    ends, acc, target = [], 0, sum(p.numel() for p in params) / groups
+    for k, p in enumerate(params):
+        acc += p.numel()
+        if acc >= target * (len(ends) + 1) or k == len(params) - 1:
+            ends.append(k + 1)
+    spans, start = [], 0
+    for e in ends:
+        lo = params[start].data_ptr() - flat.data_ptr()
+        hi = params[e - 1].data_ptr() - flat.data_ptr() + params[e - 1].numel() * esize
+        segs = es.segments_from_tensors(params)[start:e]
+        spans.append((lo // esize, hi // esize, es.es_plan_create(segs, plan.dtype, params[start:e])))
+        start = e
 
-    def one(t):
-        for h, p in zip(host, params):
-            p.copy_(h, non_blocking=True)
-        launches = run_step(es, plan, wl, t, n, sigma_at(t), sigma_at(t + 1), s_handle, None,
-                            fused)
-        for h, p in zip(host, params):
-            h.copy_(p, non_blocking=True)
-        return launches
+    def one(t, record):
+        seeds, rewards = generation_inputs(wl, t, n)
+        sigma, sigma_next = sigma_at(t), sigma_at(t + 1)
+        ev = [torch.cuda.Event(enable_timing=True) for _ in range(2)]
+        ev[0].record(stream)
+        # in: copy each group, then its first pass of the generation
+        for g, (a, b, gplan) in enumerate(spans):
+            cs = copy_streams[g % nstreams]
+            if g < nstreams:
+                cs.wait_stream(stream)
+            with torch.cuda.stream(cs):
+                flat[a:b].copy_(host[a:b], non_blocking=True)
+            stream.wait_stream(cs)
+            if fused:
+                es.es_restore_perturb(gplan, int(seeds[0]), sigma, int(seeds[1]), sigma, s_handle)
+            else:
+                es.es_perturb(gplan, int(seeds[0]), sigma, s_handle)
+        # middle of the generation on the whole plan
+        if fused:
+            for i in range(2, n):
+                es.es_restore_perturb(plan, int(seeds[i - 1]), sigma, int(seeds[i]), sigma, s_handle)
+            es.es_restore(plan, int(seeds[n - 1]), sigma, s_handle)
+        else:
+            es.es_restore(plan, int(seeds[0]), sigma, s_handle)
+            for i in range(1, n):
+                es.es_perturb(plan, int(seeds[i]), sigma, s_handle)
+                es.es_restore(plan, int(seeds[i]), sigma, s_handle)
+        coeffs = es.es_update_coeffs(es.es_normalize_rewards(rewards, 1e-8), wl.alpha, sigma,
+                                     es.ES_SCALE_PAPER)
+        first_next = int(generation_inputs(wl, t + 1, n)[0][0])
+        # out: last pass per group, then copy it back
+        for g, (a, b, gplan) in enumerate(spans):
+            if fused:
+                es.es_update_perturb(gplan, seeds, coeffs, first_next, sigma_next, s_handle)
+            else:
+                es.es_update(gplan, seeds, coeffs, s_handle)
+            cs = copy_streams[g % nstreams]
+            cs.wait_stream(stream)
+            with torch.cuda.stream(cs):
+                host[a:b].copy_(flat[a:b], non_blocking=True)
+        for cs in copy_streams:
+            stream.wait_stream(cs)
+        ev[1].record(stream)
+        if record is not None:
+            record.append(ev)
 
-    one(0)
+    one(0, None)
     torch.cuda.synchronize()
     barrier(dist)
+    evs = []
     e0 = torch.cuda.Event(enable_timing=True)
     e1 = torch.cuda.Event(enable_timing=True)
     e0.record(stream)
     for k in range(args.e2e_steps):
-        one(args.warmup + k)
+        one(args.warmup + k, evs)
     e1.record(stream)
     torch.cuda.synchronize()
     ms = max_over_ranks(e0.elapsed_time(e1), dist)
+    for _, _, gplan in spans:
+        gplan.close()
     P = sum(p.numel() for p in params)
     del host
     return {"value": world * P * n * args.e2e_steps / (ms / 1e3), "unit": UNIT,
             "steps": args.e2e_steps, "ms_per_step": ms / args.e2e_steps,
-            "h2d_bytes_per_step": bytes_per_copy, "d2h_bytes_per_step": bytes_per_copy}
+            "h2d_bytes_per_step": bytes_per_copy, "d2h_bytes_per_step": bytes_per_copy,
+            "layout": f"one pinned host buffer and one device buffer holding every tensor; "
+                      f"{len(spans)} groups with a plan each, copies over {nstreams} streams "
+                      f"overlapping the first and last pass of each generation"}
 
 
 # --- CPU oracle (cpu_baseline leg and the reference arm) ---------------------------------

@@ -163,6 +163,38 @@ def init_params_torch(specs: List[TensorSpec], dtype, device, seed: int = 0, std
     return out
 
 
+def flat_offsets(specs: List[TensorSpec], align: int = 8) -> List[int]:
+    """Element offsets of the tensors packed in one buffer, each rounded up to a
+    multiple of `align` elements (16 bytes for bf16 at align 8); the last entry
+    is the buffer length."""
+    offs, pos = [], 0
+    for s in specs:
+        offs.append(pos)
+        pos = (pos + s.numel + align - 1) // align * align
+    offs.append(pos)
+    return offs
+
+
+def init_params_flat(specs: List[TensorSpec], dtype, device, seed: int = 0, std: float = 0.02):
+    """The parameter set in one allocation: returns (flat buffer, one view per
+    spec). Views start at 16-byte aligned offsets; the padding between them is
+    zero and belongs to no tensor. Values as in init_params_torch."""
+    import torch
+    offs = flat_offsets(specs)
+    flat = torch.zeros(offs[-1], dtype=dtype, device=device)
+    gen = torch.Generator(device=device)
+    gen.manual_seed(seed)
+    views = []
+    for s, o in zip(specs, offs):
+        t = flat[o:o + s.numel]
+        if s.kind == "norm":
+            t.fill_(1.0)
+        else:
+            t.normal_(0.0, std, generator=gen)
+        views.append(t)
+    return flat, views
+
+
 def sample_offsets(numel: int, n_random: int, seed: int, edge: int = 64) -> np.ndarray:
     """Sorted unique local offsets: the first and last `edge` elements of a
     tensor plus `n_random` uniform ones (parity checks at full size)."""
