@@ -266,10 +266,17 @@ def gauss_per_elem(kind, n):
     if kind in GAUSS_PER_ELEM:
         return GAUSS_PER_ELEM[kind]
     return n + 1 if kind == "update_perturb" else n
-# Philox4x32-10: 10 rounds x 2 products of 32x32->64 bits per 4 outputs, each
-# product two 32-bit multiplies (high and low word): 10 per Gaussian.
-IMUL_PER_GAUSS = 10
+# Philox4x32-10 on counter (j_lo, j_hi, 0, 0): 10 rounds x 2 products of
+# 32x32->64 bits per 4 outputs, less the first round's product by 0 and the
+# second round's product of (key, j_hi) alone (shared by a tile): 18 products,
+# each two 32-bit multiplies (high and low word), i.e. 9 per Gaussian.
+IMUL_PER_GAUSS = 9
 IMUL_PER_CLK_SM = 64
+# Box-Muller: log2, sqrt, sin and cos per pair on the MUFU pipe (16 per clock
+# per SM): 2 per Gaussian. On sm_103a the integer-multiply and MUFU work of one
+# SM sub-partition does not overlap (measured), so their times add.
+MUFU_PER_GAUSS = 2
+MUFU_PER_CLK_SM = 16
 
 
 def traffic_per_element(kind):
@@ -345,6 +352,8 @@ def run_ours(args, rank, world, dist):
     sms = torch.cuda.get_device_properties(dev_index).multi_processor_count
     imul_peak = sms * IMUL_PER_CLK_SM * sm_max_mhz * 1e6          # 32-bit multiplies / s
     gauss_peak = imul_peak / IMUL_PER_GAUSS
+    shared_peak = sms * sm_max_mhz * 1e6 / (IMUL_PER_GAUSS / IMUL_PER_CLK_SM +
+                                             MUFU_PER_GAUSS / MUFU_PER_CLK_SM)
     bytes_per_launch = 2 * esize * P
     kernels = {}
     for name in timers.names():
@@ -356,7 +365,8 @@ def run_ours(args, rank, world, dist):
         kernels[name] = {"kernel": KERNEL_NAME[name], "launches": timers.count(name),
                          "mean_ms": mean, "share": timers.total_ms(name) / ms,
                          "gbs": gbs, "gauss_per_s": gps, "hbm_frac": hbm_frac,
-                         "alu_frac": alu_frac, "bound": "alu" if alu_frac > hbm_frac else "hbm"}
+                         "alu_frac": alu_frac, "imul_mufu_frac": gps / shared_peak,
+                         "bound": "alu" if alu_frac > hbm_frac else "hbm"}
     dom = max(kernels, key=lambda k: kernels[k]["share"])
     d = kernels[dom]
     tpe = traffic_per_element(dom)
@@ -371,6 +381,11 @@ def run_ours(args, rank, world, dist):
                 "traffic": traffic,
                 "peak_source": f"{sms} SMs x {IMUL_PER_CLK_SM} 32-bit integer multiplies/clk x "
                                f"{sm_max_mhz:.0f} MHz; {IMUL_PER_GAUSS} multiplies per Gaussian"}
+    roof["imul_mufu_bound"] = {
+        "gauss_per_s": shared_peak, "frac": d["gauss_per_s"] / shared_peak,
+        "source": f"integer-multiply and MUFU work issue from the same SM sub-partition "
+                  f"without overlap: {IMUL_PER_GAUSS}/{IMUL_PER_CLK_SM} + "
+                  f"{MUFU_PER_GAUSS}/{MUFU_PER_CLK_SM} SM-clocks per Gaussian"}
     roof.update({"kernel": d["kernel"], "hbm_frac": d["hbm_frac"], "alu_frac": d["alu_frac"],
                  "algorithmic_bytes_per_launch": bytes_per_launch,
                  "gaussians_per_launch": gauss_per_elem(dom, n) * P})
