@@ -326,3 +326,53 @@ def test_replay_argument_errors(es):
         es.es_update_perturb(plan, [1], [1.0], 2, float("nan"))
     assert ei.value.status == es.ES_ERR_NONFINITE
     plan.close()
+
+
+@pytest.mark.parametrize("dtype", ["bf16", "f32"])
+def test_results_do_not_depend_on_the_work_distribution(es, dtype):
+    # The same tensors (same index bases) in plans that list them in different
+    # orders give different tile-to-CTA assignments; every element must come
+    # out bit-identical all the same.
+    numels = [100003, 7, 8192 * 5 + 3, 2560, 65536, 9]
+    a = make_params(dtype, numels, seed=14)
+    b = [t.clone() for t in a]
+    bases = [s.index_base for s in es.segments_from_tensors(a)]
+    plan_a = es.plan_from_tensors(a, bases)
+    order = [3, 0, 5, 2, 4, 1]
+    plan_b = es.plan_from_tensors([b[k] for k in order], [bases[k] for k in order])
+    seeds = np.arange(40, 52, dtype=np.uint64)
+    coeffs = np.linspace(-1e-3, 1e-3, 12).astype(np.float32)
+    for p in (plan_a, plan_b):
+        es.es_perturb(p, 5, 1e-3)
+        es.es_restore_perturb(p, 5, 1e-3, 6, 1e-3)
+        es.es_update_perturb(p, seeds, coeffs, 7, 1e-3)
+        es.es_replay(p, seeds, coeffs, [5, 7])
+    torch.cuda.synchronize()
+    for x, y in zip(a, b):
+        assert torch.equal(_int_view(x), _int_view(y))
+    plan_a.close()
+    plan_b.close()
+
+
+def test_many_tiny_segments(es, oracle):
+    # 2000 segments of 1..40 elements with gaps in index space: thousands of
+    # ragged one-tile segments, each CTA walking far through the table.
+    rng = np.random.default_rng(15)
+    numels = [int(n) for n in rng.integers(1, 41, size=2000)]
+    tensors = make_params("bf16", numels, seed=16)
+    bases, pos = [], 0
+    for n in numels:
+        bases.append(pos)
+        pos += (n + 7) // 8 * 8 + 8 * int(rng.integers(0, 3))
+    plan, segs = build_plan(es, tensors, bases)
+    before = [host_values(t) for t in tensors]
+    seeds = np.array([3, 4, 5], dtype=np.uint64)
+    coeffs = np.array([1e-3, -2e-3, 5e-4], dtype=np.float32)
+    es.es_update(plan, seeds, coeffs)
+    torch.cuda.synchronize()
+    g = np.concatenate(indices(segs))
+    got = np.concatenate([host_values(t) for t in tensors])
+    want = oracle.update(np.concatenate(before), g, seeds, coeffs, "bf16")
+    tol = noise_abs_tol([oracle.noise_at(int(s), g) for s in seeds], coeffs)
+    compare("bf16", got, want, "2000 tiny segments", tol)
+    plan.close()
