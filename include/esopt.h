@@ -26,9 +26,11 @@
  *   with r01 = sqrt(-2 ln u(x0)) and r23 = sqrt(-2 ln u(x2)) (Box-Muller).
  *
  * Device values are computed in fp32 and agree with the exact definition to
- * |delta eps| <= 1e-5 * max(1, |eps|). Every device entry point computes eps
- * bit-identically, so es_restore undoes es_perturb up to the storage rounding
- * and es_update uses the same directions that were evaluated.
+ * |delta eps| <= 1e-5 * max(1, |eps|). Every device entry point derives eps
+ * from bit-identical radius and angle values, and applies a scale s as
+ * fma(-(s * r), cos, theta) (resp. sin), so es_restore adds exactly the
+ * negation of es_perturb's increment (it undoes it up to the storage
+ * rounding) and es_update uses the same directions that were evaluated.
  *
  * Conventions for every function:
  *   - All device memory (parameters, noise buffers) belongs to the caller. The

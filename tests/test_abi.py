@@ -145,3 +145,21 @@ def test_product_path_has_no_cpu_fallback(E, monkeypatch, tmp_path):
     with pytest.raises(RuntimeError):
         fresh.es_sigma_cosine(1.0, 0.0, 0, 1)
     importlib.reload(mod)
+
+
+def test_noalloc_validation_rejects_before_touching_the_device(E):
+    S = E.Segment
+    cases = [
+        ([S(0x1000, 16, 0)] * (E.ES_STATIC_MAX_SEGMENTS + 1), E.ES_ERR_INVALID_ARG),
+        ([S(0x1008, 16, 0)], E.ES_ERR_ALIGNMENT),
+        ([S(0x1000, 16, 4)], E.ES_ERR_ALIGNMENT),
+        ([S(0x1000, 16, 0), S(0x1010, 16, 16)], E.ES_ERR_OVERLAP),
+        ([S(0x1000, 16, 0), S(0x2000, 16, 8)], E.ES_ERR_OVERLAP),
+    ]
+    for segs, want in cases:
+        with pytest.raises(E.EsError) as ei:
+            E.es_perturb_noalloc(segs, E.ES_BF16, 1, 1e-3)
+        assert ei.value.status == want
+    with pytest.raises(E.EsError) as ei:
+        E.es_perturb_noalloc([S(0x1000, 16, 0)], E.ES_BF16, 1, float("nan"))
+    assert ei.value.status == E.ES_ERR_NONFINITE

@@ -88,3 +88,12 @@ def test_noise_is_a_function_of_seed_and_index_only(oracle):
     base = 4 * 2**32 - 6
     seg = oracle.noise_fill(8, base, 12)
     assert np.array_equal(seg, oracle.noise_at(8, np.arange(base, base + 12, dtype=np.uint64)))
+
+
+def test_box_muller_fill_matches_the_noise_of_the_same_words(oracle):
+    # The word-pair form (reference of the exhaustive GPU transform test) pairs
+    # and orders its inputs exactly as the noise of a Philox block does.
+    for seed, j in [(3, 0), (99, 7), (2**50 + 1, 2**33 + 5)]:
+        x = oracle.noise_block(seed, j)
+        got = oracle.box_muller(np.array([x[0], x[1], x[2], x[3]], dtype=np.uint32))
+        assert np.array_equal(got, oracle.noise_fill(seed, 4 * j, 4))
