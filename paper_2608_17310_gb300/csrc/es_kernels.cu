@@ -189,58 +189,59 @@ __device__ __forceinline__ TileRef<Io> tile_ref(const SegDesc* __restrict__ segs
 }
 
 // One tile of the perturb/restore pass (kTwo: fused restore + perturb; kSame:
-// both steps use one seed, whose noise is generated once). v[u] holds the
-// thread's full vectors of the tile.
+// both steps use one seed, whose noise is generated once). The thread's
+// kVecsPerThread vectors go in passes of ES_AXPY_GROUP: each pass loads its
+// vectors, adds the noise and stores them.
 template <class Io, bool kTwo, bool kSame, bool kUniformHi>
-__device__ __forceinline__ void axpy_tile(const TileRef<Io>& r, const uint4 (&v)[kVecsPerThread],
-                                          PhiloxKey key, float scale, PhiloxKey key2,
-                                          float scale2) {
+__device__ __forceinline__ void axpy_tile(const TileRef<Io>& r, PhiloxKey key, float scale,
+                                          PhiloxKey key2, float scale2) {
   constexpr int V = Io::kVec;
+  constexpr int G = ES_AXPY_GROUP;
+  static_assert(kVecsPerThread % G == 0, "group size divides the vectors per thread");
   typename Io::Scalar* const base = r.base;
   const uint64_t numel = r.numel, index_base = r.index_base, t0 = r.t0;
   const uint32_t j_hi = static_cast<uint32_t>((index_base + t0) >> 34);
   const auto gen = make_gen<kUniformHi>(key, j_hi);
   const auto gen2 = make_gen<kUniformHi && kTwo && !kSame>(key2, j_hi);
+#pragma unroll 1
+  for (int u0 = 0; u0 < kVecsPerThread; u0 += G) {
+    uint4 v[G];
 #pragma unroll
-  for (int u = 0; u < kVecsPerThread; ++u) {
-    const uint64_t e = t0 + static_cast<uint64_t>(u * kBlockThreads + threadIdx.x) * V;
-    if (e >= numel) continue;
-    const bool full = e + V <= numel;
-    const int rem = full ? V : static_cast<int>(numel - e);
-    float f[V];
-    if (full) {
-      Io::unpack(v[u], f);
-    } else {  // ragged end of a segment
-#pragma unroll
-      for (int k = 0; k < V; ++k) f[k] = k < rem ? Io::to_f32(base[e + k]) : 0.0f;
+    for (int q = 0; q < G; ++q) {
+      const uint64_t e = t0 + static_cast<uint64_t>((u0 + q) * kBlockThreads + threadIdx.x) * V;
+      if (e + V <= numel) v[q] = *reinterpret_cast<const uint4*>(base + e);
     }
-    if (kSame) {
-      add_scaled_noise_twice<Io, V>(gen, index_base + e, scale, scale2, f);
-    } else {
-      add_scaled_noise<V>(gen, index_base + e, scale, f);
-      if (kTwo) {
-        Io::round_trip(f);
-        add_scaled_noise<V>(gen2, index_base + e, scale2, f);
+#pragma unroll
+    for (int q = 0; q < G; ++q) {
+      const uint64_t e = t0 + static_cast<uint64_t>((u0 + q) * kBlockThreads + threadIdx.x) * V;
+      if (e >= numel) continue;
+      const bool full = e + V <= numel;
+      const int rem = full ? V : static_cast<int>(numel - e);
+      float f[V];
+      if (full) {
+        Io::unpack(v[q], f);
+      } else {  // ragged end of a segment
+#pragma unroll
+        for (int k = 0; k < V; ++k) f[k] = k < rem ? Io::to_f32(base[e + k]) : 0.0f;
+      }
+      if (kSame) {
+        add_scaled_noise_twice<Io, V>(gen, index_base + e, scale, scale2, f);
+      } else {
+        add_scaled_noise<V>(gen, index_base + e, scale, f);
+        if (kTwo) {
+          Io::round_trip(f);
+          add_scaled_noise<V>(gen2, index_base + e, scale2, f);
+        }
+      }
+      if (full) {
+        *reinterpret_cast<uint4*>(base + e) = Io::pack(f);
+      } else {
+#pragma unroll
+        for (int k = 0; k < V; ++k)
+          if (k < rem) base[e + k] = Io::from_f32(f[k]);
       }
     }
-    if (full) {
-      *reinterpret_cast<uint4*>(base + e) = Io::pack(f);
-    } else {
-#pragma unroll
-      for (int k = 0; k < V; ++k)
-        if (k < rem) base[e + k] = Io::from_f32(f[k]);
-    }
   }
-}
-
-template <class Io, bool kTwo, bool kSame>
-__device__ __forceinline__ void axpy_dispatch(const TileRef<Io>& r, const uint4 (&v)[kVecsPerThread],
-                                              uint64_t tile_elems, PhiloxKey key, float scale,
-                                              PhiloxKey key2, float scale2) {
-  if (uniform_hi(r.index_base, r.t0, tile_elems, r.numel))
-    axpy_tile<Io, kTwo, kSame, true>(r, v, key, scale, key2, scale2);
-  else
-    axpy_tile<Io, kTwo, kSame, false>(r, v, key, scale, key2, scale2);
 }
 
 // theta[g] <- round(theta[g] + scale * eps_seed[g]) over every segment; with
@@ -252,18 +253,14 @@ template <class Io, bool kTwo, bool kSame>
 __global__ void ES_AXPY_BOUNDS
 axpy_noise_kernel(const SegDesc* __restrict__ segs, uint64_t total_tiles, PhiloxKey key,
                   float scale, PhiloxKey key2, float scale2) {
-  constexpr int V = Io::kVec;
-  constexpr uint64_t kTile = static_cast<uint64_t>(kBlockThreads) * kVecsPerThread * V;
+  constexpr uint64_t kTile = static_cast<uint64_t>(kBlockThreads) * kVecsPerThread * Io::kVec;
   int seg = 0;
   for (uint64_t tile = blockIdx.x; tile < total_tiles; tile += gridDim.x) {
     const TileRef<Io> cur = tile_ref<Io>(segs, seg, tile, kTile);
-    uint4 v[kVecsPerThread];
-#pragma unroll
-    for (int u = 0; u < kVecsPerThread; ++u) {
-      const uint64_t e = cur.t0 + static_cast<uint64_t>(u * kBlockThreads + threadIdx.x) * V;
-      if (e + V <= cur.numel) v[u] = *reinterpret_cast<const uint4*>(cur.base + e);
-    }
-    axpy_dispatch<Io, kTwo, kSame>(cur, v, kTile, key, scale, key2, scale2);
+    if (uniform_hi(cur.index_base, cur.t0, kTile, cur.numel))
+      axpy_tile<Io, kTwo, kSame, true>(cur, key, scale, key2, scale2);
+    else
+      axpy_tile<Io, kTwo, kSame, false>(cur, key, scale, key2, scale2);
   }
 }
 
@@ -277,56 +274,60 @@ __device__ __forceinline__ void update_tile_single(typename Io::Scalar* base, ui
                                                    const UpdateArgs& args, const PhiloxKey* s_key,
                                                    const float* s_coeff) {
   constexpr int V = Io::kVec;
+  constexpr int G = kUpdateGroup;
   const uint32_t j_hi = static_cast<uint32_t>((index_base + t0) >> 34);
   const int n = args.n;
-  uint4 v[kVecsPerThread];
-#pragma unroll
-  for (int u = 0; u < kVecsPerThread; ++u) {
-    const uint64_t e = t0 + static_cast<uint64_t>(u * kBlockThreads + threadIdx.x) * V;
-    if (e + V <= numel) v[u] = *reinterpret_cast<const uint4*>(base + e);
-  }
-  float acc[kVecsPerThread][V];
-#pragma unroll
-  for (int u = 0; u < kVecsPerThread; ++u)
-#pragma unroll
-    for (int k = 0; k < V; ++k) acc[u][k] = 0.0f;
-#pragma unroll 1
-  for (int i = 0; i < n; ++i) {
-    const auto gen = make_gen<kUniformHi>(s_key[i], j_hi);
-    const float c = s_coeff[i];
-#pragma unroll
-    for (int u = 0; u < kVecsPerThread; ++u) {
-      const uint64_t e = t0 + static_cast<uint64_t>(u * kBlockThreads + threadIdx.x) * V;
-      if (e >= numel) continue;
-      add_scaled_noise<V>(gen, index_base + e, c, acc[u]);
-    }
-  }
   const auto pgen = make_gen<kUniformHi && kPerturb>(PhiloxKey{args.pkey[0], args.pkey[1]}, j_hi);
+#pragma unroll 1
+  for (int u0 = 0; u0 < kVecsPerThread; u0 += G) {
+    uint4 v[G];
 #pragma unroll
-  for (int u = 0; u < kVecsPerThread; ++u) {
-    const uint64_t e = t0 + static_cast<uint64_t>(u * kBlockThreads + threadIdx.x) * V;
-    if (e >= numel) continue;
-    const bool full = e + V <= numel;
-    const int rem = full ? V : static_cast<int>(numel - e);
-    float f[V];
-    if (full) {
-      Io::unpack(v[u], f);
-    } else {
+    for (int q = 0; q < G; ++q) {
+      const uint64_t e = t0 + static_cast<uint64_t>((u0 + q) * kBlockThreads + threadIdx.x) * V;
+      if (e + V <= numel) v[q] = *reinterpret_cast<const uint4*>(base + e);
+    }
+    float acc[G][V];
 #pragma unroll
-      for (int k = 0; k < V; ++k) f[k] = k < rem ? Io::to_f32(base[e + k]) : 0.0f;
+    for (int q = 0; q < G; ++q)
+#pragma unroll
+      for (int k = 0; k < V; ++k) acc[q][k] = 0.0f;
+#pragma unroll 1
+    for (int i = 0; i < n; ++i) {
+      const auto gen = make_gen<kUniformHi>(s_key[i], j_hi);
+      const float c = s_coeff[i];
+#pragma unroll
+      for (int q = 0; q < G; ++q) {
+        const uint64_t e = t0 + static_cast<uint64_t>((u0 + q) * kBlockThreads + threadIdx.x) * V;
+        if (e >= numel) continue;
+        add_scaled_noise<V>(gen, index_base + e, c, acc[q]);
+      }
     }
 #pragma unroll
-    for (int k = 0; k < V; ++k) f[k] = f[k] + acc[u][k];
-    if (kPerturb) {
-      Io::round_trip(f);
-      add_scaled_noise<V>(pgen, index_base + e, args.pscale, f);
-    }
-    if (full) {
-      *reinterpret_cast<uint4*>(base + e) = Io::pack(f);
-    } else {
+    for (int q = 0; q < G; ++q) {
+      const uint64_t e = t0 + static_cast<uint64_t>((u0 + q) * kBlockThreads + threadIdx.x) * V;
+      if (e >= numel) continue;
+      const bool full = e + V <= numel;
+      const int rem = full ? V : static_cast<int>(numel - e);
+      float f[V];
+      if (full) {
+        Io::unpack(v[q], f);
+      } else {
 #pragma unroll
-      for (int k = 0; k < V; ++k)
-        if (k < rem) base[e + k] = Io::from_f32(f[k]);
+        for (int k = 0; k < V; ++k) f[k] = k < rem ? Io::to_f32(base[e + k]) : 0.0f;
+      }
+#pragma unroll
+      for (int k = 0; k < V; ++k) f[k] = f[k] + acc[q][k];
+      if (kPerturb) {
+        Io::round_trip(f);
+        add_scaled_noise<V>(pgen, index_base + e, args.pscale, f);
+      }
+      if (full) {
+        *reinterpret_cast<uint4*>(base + e) = Io::pack(f);
+      } else {
+#pragma unroll
+        for (int k = 0; k < V; ++k)
+          if (k < rem) base[e + k] = Io::from_f32(f[k]);
+      }
     }
   }
 }
@@ -341,64 +342,68 @@ __device__ __forceinline__ void update_tile(typename Io::Scalar* base, uint64_t 
                                             const UpdateArgs& args, const PhiloxKey* s_key,
                                             const float* s_coeff, const uint16_t* s_gen_end) {
   constexpr int V = Io::kVec;
+  constexpr int G = kUpdateGroup;
   const uint32_t j_hi = static_cast<uint32_t>((index_base + t0) >> 34);
-  uint4 v[kVecsPerThread];
-#pragma unroll
-  for (int u = 0; u < kVecsPerThread; ++u) {
-    const uint64_t e = t0 + static_cast<uint64_t>(u * kBlockThreads + threadIdx.x) * V;
-    if (e + V <= numel)
-      v[u] = *reinterpret_cast<const uint4*>(base + e);
-    else if (e < numel)
-      v[u] = Io::load_partial(base, e, static_cast<int>(numel - e));
-  }
-  int i = 0;
 #pragma unroll 1
-  for (int g = 0; g < args.n_gen; ++g) {
-    float acc[kVecsPerThread][V];
+  for (int u0 = 0; u0 < kVecsPerThread; u0 += G) {
+    uint4 v[G];
 #pragma unroll
-    for (int u = 0; u < kVecsPerThread; ++u)
-#pragma unroll
-      for (int k = 0; k < V; ++k) acc[u][k] = 0.0f;
-    const int end = s_gen_end[g];
+    for (int q = 0; q < G; ++q) {
+      const uint64_t e = t0 + static_cast<uint64_t>((u0 + q) * kBlockThreads + threadIdx.x) * V;
+      if (e + V <= numel)
+        v[q] = *reinterpret_cast<const uint4*>(base + e);
+      else if (e < numel)
+        v[q] = Io::load_partial(base, e, static_cast<int>(numel - e));
+    }
+    int i = 0;
 #pragma unroll 1
-    for (; i < end; ++i) {
-      const auto gen = make_gen<kUniformHi>(s_key[i], j_hi);
-      const float c = s_coeff[i];
+    for (int g = 0; g < args.n_gen; ++g) {
+      float acc[G][V];
 #pragma unroll
-      for (int u = 0; u < kVecsPerThread; ++u) {
-        const uint64_t e = t0 + static_cast<uint64_t>(u * kBlockThreads + threadIdx.x) * V;
+      for (int q = 0; q < G; ++q)
+#pragma unroll
+        for (int k = 0; k < V; ++k) acc[q][k] = 0.0f;
+      const int end = s_gen_end[g];
+#pragma unroll 1
+      for (; i < end; ++i) {
+        const auto gen = make_gen<kUniformHi>(s_key[i], j_hi);
+        const float c = s_coeff[i];
+#pragma unroll
+        for (int q = 0; q < G; ++q) {
+          const uint64_t e = t0 + static_cast<uint64_t>((u0 + q) * kBlockThreads + threadIdx.x) * V;
+          if (e >= numel) continue;
+          add_scaled_noise<V>(gen, index_base + e, c, acc[q]);
+        }
+      }
+#pragma unroll
+      for (int q = 0; q < G; ++q) {
+        float f[V];
+        Io::unpack(v[q], f);
+#pragma unroll
+        for (int k = 0; k < V; ++k) f[k] = f[k] + acc[q][k];
+        v[q] = Io::pack(f);
+      }
+    }
+    if (args.perturb) {
+      const auto gen = make_gen<kUniformHi>(PhiloxKey{args.pkey[0], args.pkey[1]}, j_hi);
+#pragma unroll
+      for (int q = 0; q < G; ++q) {
+        const uint64_t e = t0 + static_cast<uint64_t>((u0 + q) * kBlockThreads + threadIdx.x) * V;
         if (e >= numel) continue;
-        add_scaled_noise<V>(gen, index_base + e, c, acc[u]);
+        float f[V];
+        Io::unpack(v[q], f);
+        add_scaled_noise<V>(gen, index_base + e, args.pscale, f);
+        v[q] = Io::pack(f);
       }
     }
 #pragma unroll
-    for (int u = 0; u < kVecsPerThread; ++u) {
-      float f[V];
-      Io::unpack(v[u], f);
-#pragma unroll
-      for (int k = 0; k < V; ++k) f[k] = f[k] + acc[u][k];
-      v[u] = Io::pack(f);
+    for (int q = 0; q < G; ++q) {
+      const uint64_t e = t0 + static_cast<uint64_t>((u0 + q) * kBlockThreads + threadIdx.x) * V;
+      if (e + V <= numel)
+        *reinterpret_cast<uint4*>(base + e) = v[q];
+      else if (e < numel)
+        Io::store_partial(base, e, static_cast<int>(numel - e), v[q]);
     }
-  }
-  if (args.perturb) {
-    const auto gen = make_gen<kUniformHi>(PhiloxKey{args.pkey[0], args.pkey[1]}, j_hi);
-#pragma unroll
-    for (int u = 0; u < kVecsPerThread; ++u) {
-      const uint64_t e = t0 + static_cast<uint64_t>(u * kBlockThreads + threadIdx.x) * V;
-      if (e >= numel) continue;
-      float f[V];
-      Io::unpack(v[u], f);
-      add_scaled_noise<V>(gen, index_base + e, args.pscale, f);
-      v[u] = Io::pack(f);
-    }
-  }
-#pragma unroll
-  for (int u = 0; u < kVecsPerThread; ++u) {
-    const uint64_t e = t0 + static_cast<uint64_t>(u * kBlockThreads + threadIdx.x) * V;
-    if (e + V <= numel)
-      *reinterpret_cast<uint4*>(base + e) = v[u];
-    else if (e < numel)
-      Io::store_partial(base, e, static_cast<int>(numel - e), v[u]);
   }
 }
 

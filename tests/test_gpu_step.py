@@ -376,3 +376,64 @@ def test_many_tiny_segments(es, oracle):
     tol = noise_abs_tol([oracle.noise_at(int(s), g) for s in seeds], coeffs)
     compare("bf16", got, want, "2000 tiny segments", tol)
     plan.close()
+
+
+def test_segment_larger_than_2_to_32_elements(es, oracle):
+    # One 8.6 GB bf16 segment: element offsets inside it pass 2^32, and its
+    # global indices cross a 2^34 boundary (index base chosen so).
+    n = 2**32 + 8200
+    t = torch.empty(n, dtype=torch.bfloat16, device="cuda")
+    t.normal_(0.0, 0.02, generator=torch.Generator(device="cuda").manual_seed(3))
+    base = 2**34 - 8 * 1000
+    plan = es.es_plan_create([es.Segment(t.data_ptr(), n, base)], es.ES_BF16, [t])
+    offs = np.unique(np.concatenate([np.arange(0, 64), np.arange(8000 - 64, 8000 + 64),
+                                     np.arange(2**32 - 64, 2**32 + 64), np.arange(n - 64, n),
+                                     np.random.default_rng(4).integers(0, n, 20000)])).astype(np.int64)
+    idx = torch.from_numpy(offs).cuda()
+    g = (np.uint64(base) + offs.astype(np.uint64))
+    before = t.index_select(0, idx).view(torch.int16).cpu().numpy().view(np.uint16)
+    es.es_perturb(plan, 77, 1e-3)
+    torch.cuda.synchronize()
+    got = t.index_select(0, idx).view(torch.int16).cpu().numpy().view(np.uint16)
+    tol = noise_abs_tol([oracle.noise_at(77, g)], [1e-3])
+    compare("bf16", got, oracle.perturb(before, g, 77, 1e-3, "bf16"), "2^32+ segment perturb", tol)
+    seeds, coeffs = np.array([5, 6], np.uint64), np.array([1e-3, -1e-3], np.float32)
+    es.es_update(plan, seeds, coeffs)
+    torch.cuda.synchronize()
+    after = t.index_select(0, idx).view(torch.int16).cpu().numpy().view(np.uint16)
+    tol = noise_abs_tol([oracle.noise_at(int(s), g) for s in seeds], coeffs)
+    compare("bf16", after, oracle.update(got, g, seeds, coeffs, "bf16"), "2^32+ segment update", tol)
+    plan.close()
+    del t
+    torch.cuda.empty_cache()
+
+
+@pytest.mark.parametrize("dtype", ["bf16", "f32"])
+def test_special_values(es, oracle, dtype):
+    # inf stays inf, NaN stays NaN, signed zeros, subnormals and the largest
+    # finite values go through the same rounding as on the oracle.
+    fmax = 3.3895313892515355e38 if dtype == "bf16" else float(np.finfo(np.float32).max)
+    vals = np.array([np.inf, -np.inf, np.nan, 0.0, -0.0, 1e-40, -1e-40, 1e-45, fmax, -fmax,
+                     1.0, -2.0, 3e38, 6e-39] * 16, dtype=np.float32)
+    t = torch.from_numpy(vals.copy())
+    t = (t.to(torch.bfloat16) if dtype == "bf16" else t).cuda()
+    plan, segs = build_plan(es, [t])
+    before = host_values(t)
+    g = indices(segs)[0]
+    es.es_perturb(plan, 9, 0.5)
+    torch.cuda.synchronize()
+    got = host_values(t)
+    want = oracle.perturb(before, g, 9, 0.5, dtype)
+    if dtype == "bf16":
+        gv = (got.astype(np.uint32) << 16).view(np.float32)
+        wv = (want.astype(np.uint32) << 16).view(np.float32)
+    else:
+        gv, wv = got, want
+    nan = np.isnan(wv)
+    assert np.array_equal(np.isnan(gv), nan)
+    inf = np.isinf(wv)
+    assert np.array_equal(gv[inf], wv[inf])
+    fin = ~nan & ~inf
+    tol = noise_abs_tol([oracle.noise_at(9, g)], [0.5])[fin]
+    compare(dtype, got[fin], want[fin], f"special values {dtype}", tol)
+    plan.close()
