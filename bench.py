@@ -33,7 +33,8 @@ from paper_2608_17310_gb300 import inputs as I  # noqa: E402
 
 METRIC = "ES step param*seed/s (perturb+restore+update) and % of HBM/ALU roofline"
 UNIT = "param*seed/s"
-SIGMA_FINAL = {"qwen27b": 2.5e-4, "qwen4b": 5e-4, "qwen4b_4layer": 5e-4, "toy": 1e-3}
+SIGMA_FINAL = {"qwen27b": 2.5e-4, "qwen4b": 5e-4, "qwen4b_f32": 5e-4, "qwen4b_4layer": 5e-4,
+               "toy": 1e-3}
 SCHEDULE_T = 100
 CPU_SAMPLE = 1 << 21
 
@@ -43,7 +44,7 @@ def parse():
     p.add_argument("--gpus", type=int, default=1)
     p.add_argument("--steps", type=int, default=5)
     p.add_argument("--warmup", type=int, default=3)
-    p.add_argument("--workload", default="qwen27b", choices=["qwen27b", "qwen4b", "qwen4b_4layer", "toy"])
+    p.add_argument("--workload", default="qwen27b", choices=["qwen27b", "qwen4b", "qwen4b_f32", "qwen4b_4layer", "toy"])
     p.add_argument("--population", type=int, default=None, help="override N")
     p.add_argument("--impl", default="ours", choices=["ours", "reference"])
     p.add_argument("--no-e2e", action="store_true")

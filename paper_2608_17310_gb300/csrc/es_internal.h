@@ -21,10 +21,6 @@ constexpr int kBlockThreads = 256;
 #ifndef ES_UPDATE_MIN_BLOCKS
 #define ES_UPDATE_MIN_BLOCKS 0
 #endif
-// Vectors the perturb/restore kernels process per pass (1, 2 or 4).
-#ifndef ES_AXPY_GROUP
-#define ES_AXPY_GROUP 4
-#endif
 #if ES_AXPY_MIN_BLOCKS > 0
 #define ES_AXPY_BOUNDS __launch_bounds__(esopt::kBlockThreads, ES_AXPY_MIN_BLOCKS)
 #else
@@ -35,13 +31,11 @@ constexpr int kBlockThreads = 256;
 #else
 #define ES_UPDATE_BOUNDS __launch_bounds__(esopt::kBlockThreads)
 #endif
-// 16-byte vectors per thread per tile.
-#ifndef ES_VECS_PER_THREAD
-#define ES_VECS_PER_THREAD 4
-#endif
-constexpr int kVecsPerThread = ES_VECS_PER_THREAD;
-// Vectors the update kernel accumulates at a time (its fp32 accumulators).
-constexpr int kUpdateGroup = kVecsPerThread < 4 ? kVecsPerThread : 4;
+// 16-byte vectors each thread owns per tile. All of them are processed in one
+// pass: the independent Philox chains (ILP) matter more than occupancy here
+// (measured: splitting into passes of 1 or 2 vectors, or 8 vectors per
+// thread, were slower).
+constexpr int kVecsPerThread = 4;
 // Elements per 16-byte vector, per dtype.
 constexpr int vec_elems(es_dtype_t dt) { return dt == ES_BF16 ? 8 : 4; }
 // Elements per tile: a tile is the unit one CTA processes at a time; tiles

@@ -2,10 +2,11 @@
 // the fused N-seed update (theta += sum_i c_i eps_i), plus a noise fill.
 //
 // All three stream the parameter set once per launch. Work is cut into tiles
-// of kBlockThreads * kVecsPerThread 16-byte vectors that never straddle a
-// segment; persistent CTAs walk the tiles in grid-stride order, so consecutive
-// CTAs touch consecutive memory and each CTA advances through the segment table
-// monotonically (one table lookup per tile, no per-element search).
+// of kBlockThreads threads x kVecsPerThread 16-byte vectors that never
+// straddle a segment; persistent CTAs walk the tiles in grid-stride
+// order, so consecutive CTAs touch consecutive memory and each CTA advances
+// through the segment table monotonically (one table lookup per tile, no
+// per-element search).
 // Every element is owned by exactly one thread: no atomics, no shared state
 // between threads except the staged seeds of the update.
 #include <cuda_bf16.h>
@@ -22,6 +23,7 @@ namespace {
 // 16-byte vector <-> fp32 registers, and single-element access for tails.
 struct Bf16Io {
   static constexpr int kVec = 8;
+  static constexpr int kVecs = kVecsPerThread;
   using Scalar = uint16_t;
   __device__ static float to_f32(uint16_t h) { return __uint_as_float(static_cast<uint32_t>(h) << 16); }
   __device__ static uint16_t from_f32(float f) { return __bfloat16_as_ushort(__float2bfloat16_rn(f)); }
@@ -67,6 +69,7 @@ struct Bf16Io {
 
 struct F32Io {
   static constexpr int kVec = 4;
+  static constexpr int kVecs = kVecsPerThread;
   using Scalar = float;
   __device__ static float to_f32(float f) { return f; }
   __device__ static float from_f32(float f) { return f; }
@@ -189,57 +192,51 @@ __device__ __forceinline__ TileRef<Io> tile_ref(const SegDesc* __restrict__ segs
 }
 
 // One tile of the perturb/restore pass (kTwo: fused restore + perturb; kSame:
-// both steps use one seed, whose noise is generated once). The thread's
-// kVecsPerThread vectors go in passes of ES_AXPY_GROUP: each pass loads its
-// vectors, adds the noise and stores them.
+// both steps use one seed, whose noise is generated once). Each thread loads
+// its vectors, adds the noise and stores them, all in one pass.
 template <class Io, bool kTwo, bool kSame, bool kUniformHi>
 __device__ __forceinline__ void axpy_tile(const TileRef<Io>& r, PhiloxKey key, float scale,
                                           PhiloxKey key2, float scale2) {
-  constexpr int V = Io::kVec;
-  constexpr int G = ES_AXPY_GROUP;
-  static_assert(kVecsPerThread % G == 0, "group size divides the vectors per thread");
+  constexpr int V = Io::kVec, U = Io::kVecs;
   typename Io::Scalar* const base = r.base;
   const uint64_t numel = r.numel, index_base = r.index_base, t0 = r.t0;
   const uint32_t j_hi = static_cast<uint32_t>((index_base + t0) >> 34);
   const auto gen = make_gen<kUniformHi>(key, j_hi);
   const auto gen2 = make_gen<kUniformHi && kTwo && !kSame>(key2, j_hi);
-#pragma unroll 1
-  for (int u0 = 0; u0 < kVecsPerThread; u0 += G) {
-    uint4 v[G];
+  uint4 v[U];
 #pragma unroll
-    for (int q = 0; q < G; ++q) {
-      const uint64_t e = t0 + static_cast<uint64_t>((u0 + q) * kBlockThreads + threadIdx.x) * V;
-      if (e + V <= numel) v[q] = *reinterpret_cast<const uint4*>(base + e);
+  for (int u = 0; u < U; ++u) {
+    const uint64_t e = t0 + static_cast<uint64_t>(u * kBlockThreads + threadIdx.x) * V;
+    if (e + V <= numel) v[u] = *reinterpret_cast<const uint4*>(base + e);
+  }
+#pragma unroll
+  for (int u = 0; u < U; ++u) {
+    const uint64_t e = t0 + static_cast<uint64_t>(u * kBlockThreads + threadIdx.x) * V;
+    if (e >= numel) continue;
+    const bool full = e + V <= numel;
+    const int rem = full ? V : static_cast<int>(numel - e);
+    float f[V];
+    if (full) {
+      Io::unpack(v[u], f);
+    } else {  // ragged end of a segment
+#pragma unroll
+      for (int k = 0; k < V; ++k) f[k] = k < rem ? Io::to_f32(base[e + k]) : 0.0f;
     }
-#pragma unroll
-    for (int q = 0; q < G; ++q) {
-      const uint64_t e = t0 + static_cast<uint64_t>((u0 + q) * kBlockThreads + threadIdx.x) * V;
-      if (e >= numel) continue;
-      const bool full = e + V <= numel;
-      const int rem = full ? V : static_cast<int>(numel - e);
-      float f[V];
-      if (full) {
-        Io::unpack(v[q], f);
-      } else {  // ragged end of a segment
-#pragma unroll
-        for (int k = 0; k < V; ++k) f[k] = k < rem ? Io::to_f32(base[e + k]) : 0.0f;
+    if (kSame) {
+      add_scaled_noise_twice<Io, V>(gen, index_base + e, scale, scale2, f);
+    } else {
+      add_scaled_noise<V>(gen, index_base + e, scale, f);
+      if (kTwo) {
+        Io::round_trip(f);
+        add_scaled_noise<V>(gen2, index_base + e, scale2, f);
       }
-      if (kSame) {
-        add_scaled_noise_twice<Io, V>(gen, index_base + e, scale, scale2, f);
-      } else {
-        add_scaled_noise<V>(gen, index_base + e, scale, f);
-        if (kTwo) {
-          Io::round_trip(f);
-          add_scaled_noise<V>(gen2, index_base + e, scale2, f);
-        }
-      }
-      if (full) {
-        *reinterpret_cast<uint4*>(base + e) = Io::pack(f);
-      } else {
+    }
+    if (full) {
+      *reinterpret_cast<uint4*>(base + e) = Io::pack(f);
+    } else {
 #pragma unroll
-        for (int k = 0; k < V; ++k)
-          if (k < rem) base[e + k] = Io::from_f32(f[k]);
-      }
+      for (int k = 0; k < V; ++k)
+        if (k < rem) base[e + k] = Io::from_f32(f[k]);
     }
   }
 }
@@ -274,12 +271,12 @@ __device__ __forceinline__ void update_tile_single(typename Io::Scalar* base, ui
                                                    const UpdateArgs& args, const PhiloxKey* s_key,
                                                    const float* s_coeff) {
   constexpr int V = Io::kVec;
-  constexpr int G = kUpdateGroup;
+  constexpr int G = Io::kVecs;
   const uint32_t j_hi = static_cast<uint32_t>((index_base + t0) >> 34);
   const int n = args.n;
   const auto pgen = make_gen<kUniformHi && kPerturb>(PhiloxKey{args.pkey[0], args.pkey[1]}, j_hi);
-#pragma unroll 1
-  for (int u0 = 0; u0 < kVecsPerThread; u0 += G) {
+  {
+    constexpr int u0 = 0;
     uint4 v[G];
 #pragma unroll
     for (int q = 0; q < G; ++q) {
@@ -342,10 +339,10 @@ __device__ __forceinline__ void update_tile(typename Io::Scalar* base, uint64_t 
                                             const UpdateArgs& args, const PhiloxKey* s_key,
                                             const float* s_coeff, const uint16_t* s_gen_end) {
   constexpr int V = Io::kVec;
-  constexpr int G = kUpdateGroup;
+  constexpr int G = Io::kVecs;
   const uint32_t j_hi = static_cast<uint32_t>((index_base + t0) >> 34);
-#pragma unroll 1
-  for (int u0 = 0; u0 < kVecsPerThread; u0 += G) {
+  {
+    constexpr int u0 = 0;
     uint4 v[G];
 #pragma unroll
     for (int q = 0; q < G; ++q) {

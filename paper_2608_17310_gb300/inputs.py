@@ -91,6 +91,10 @@ WORKLOADS = {
                        "Qwen3.5-4B-shaped bf16 (4,022,458,880 params, 326 tensors), N=16"),
     "qwen27b": Workload("qwen27b", "bf16", 30, 5e-4, 2.5e-4, "uniform",
                         "27B-shaped bf16 (22,695,777,280 params, 579 tensors), N=30"),
+    # the 4B shapes in fp32 storage (16.1 GB): the perturb pass moves 8 B per
+    # Gaussian there, so HBM rather than the generator bounds it
+    "qwen4b_f32": Workload("qwen4b_f32", "f32", 16, 1e-3, 5e-4, "bernoulli0.3",
+                           "Qwen3.5-4B-shaped fp32 (4,022,458,880 params, 326 tensors), N=16"),
     # profiling case: the 4B shapes cut to 4 layers (about 1.6 GB, larger than L2)
     "qwen4b_4layer": Workload("qwen4b_4layer", "bf16", 16, 1e-3, 5e-4, "bernoulli0.3",
                               "Qwen3.5-4B shapes, 4 layers (792,680,960 params, 38 tensors), N=16"),
@@ -98,7 +102,7 @@ WORKLOADS = {
 
 
 def shapes_for(name: str) -> List[TensorSpec]:
-    if name == "qwen4b":
+    if name in ("qwen4b", "qwen4b_f32"):
         return qwen4b_shapes()
     if name == "qwen27b":
         return qwen27b_shapes()
