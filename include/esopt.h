@@ -128,7 +128,8 @@ uint64_t es_plan_numel(es_plan_t plan);
 /*
  * Assigns index_base to each segment in order: the first gets 0, each next one
  * the previous base + numel rounded up to a multiple of 8. Returns the end of
- * the index range (the last base + numel). Host-only, pure.
+ * the index range (the last base + numel), or 0 if the range would pass 2^64
+ * (then the bases are only partly assigned). Host-only, pure.
  */
 uint64_t es_assign_index_bases(es_segment_t* segs, int nseg);
 
@@ -242,7 +243,9 @@ es_status_t es_update_perturb(es_plan_t plan, const uint64_t* seeds, const float
  * the generations back to back; counts[g] (1 .. ES_MAX_SEEDS) is the size of
  * generation g. Up to 256 generations and ES_MAX_SEEDS seeds are fused per
  * pass over theta; longer logs take several passes, split between
- * generations. Host arrays; asynchronous on `stream`.
+ * generations. Host arrays; asynchronous on `stream`. All arguments are
+ * checked before the first pass; if a launch then fails (ES_ERR_CUDA), the
+ * passes before it have been applied.
  * Errors: ES_ERR_INVALID_ARG (NULL, generations < 1, an empty generation),
  * ES_ERR_TOO_MANY_SEEDS (a generation over ES_MAX_SEEDS), ES_ERR_NONFINITE,
  * ES_ERR_WRONG_DEVICE, ES_ERR_CUDA.

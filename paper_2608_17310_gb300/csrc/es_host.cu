@@ -159,7 +159,14 @@ es_status_t es_plan_create(const es_segment_t* segs, int nseg, es_dtype_t dtype,
   }
   // No two segments may share memory or global indices: each element must have
   // one owner and one noise stream.
-  std::vector<int> order(nseg);
+  std::vector<int> order;
+  std::vector<esopt::SegDesc> table;
+  try {
+    order.resize(static_cast<size_t>(nseg));
+    table.resize(static_cast<size_t>(nseg) + 1);
+  } catch (const std::bad_alloc&) {
+    return fail(ES_ERR_NO_MEMORY, "es_plan_create: host allocation failed");
+  }
   for (int k = 0; k < nseg; ++k) order[k] = k;
   std::sort(order.begin(), order.end(),
             [&](int a, int b) { return segs[a].index_base < segs[b].index_base; });
@@ -181,7 +188,6 @@ es_status_t es_plan_create(const es_segment_t* segs, int nseg, es_dtype_t dtype,
   }
 
   const uint64_t tile = esopt::tile_elems(dtype);
-  std::vector<esopt::SegDesc> table(static_cast<size_t>(nseg) + 1);
   uint64_t tiles = 0;
   for (int k = 0; k < nseg; ++k) {
     table[k] = esopt::SegDesc{segs[k].data, segs[k].numel, segs[k].index_base, tiles};
@@ -236,6 +242,7 @@ uint64_t es_assign_index_bases(es_segment_t* segs, int nseg) {
   if (segs == nullptr || nseg < 1) return 0;
   uint64_t base = 0, end = 0;
   for (int k = 0; k < nseg; ++k) {
+    if (segs[k].numel > UINT64_MAX - 7 - base) return 0;  // the range would pass 2^64
     segs[k].index_base = base;
     end = base + segs[k].numel;
     base = (end + 7) & ~static_cast<uint64_t>(7);
@@ -396,17 +403,17 @@ es_status_t es_normalize_rewards(const double* rewards, int n, double eps_z, dou
     for (int i = 0; i < n; ++i) rhat[i] = 0.0;
     return ok();
   }
-  std::vector<double> r(rewards, rewards + n);
-  for (double& v : r)
-    if (!std::isfinite(v)) v = lo;
+  // rewards and rhat may alias: every rhat[i] is written after the last read
+  // of rewards[i].
+  auto value = [&](int i) { return std::isfinite(rewards[i]) ? rewards[i] : lo; };
   double mu = 0.0;
-  for (double v : r) mu += v;
+  for (int i = 0; i < n; ++i) mu += value(i);
   mu /= n;
   double var = 0.0;
-  for (double v : r) var += (v - mu) * (v - mu);
+  for (int i = 0; i < n; ++i) var += (value(i) - mu) * (value(i) - mu);
   var /= n;
   const double denom = std::sqrt(var) + eps_z;
-  for (int i = 0; i < n; ++i) rhat[i] = (r[i] - mu) / denom;
+  for (int i = 0; i < n; ++i) rhat[i] = (value(i) - mu) / denom;
   return ok();
 }
 

@@ -163,3 +163,19 @@ def test_noalloc_validation_rejects_before_touching_the_device(E):
     with pytest.raises(E.EsError) as ei:
         E.es_perturb_noalloc([S(0x1000, 16, 0)], E.ES_BF16, 1, float("nan"))
     assert ei.value.status == E.ES_ERR_NONFINITE
+
+
+def test_normalize_rewards_in_place(E, oracle):
+    import ctypes
+    R = np.array([0.3, np.nan, 0.9, 0.1, 0.5, 0.5])
+    want = oracle.zscore(R.copy(), 1e-8)
+    buf = R.copy()
+    P = ctypes.POINTER(ctypes.c_double)
+    st = E.lib().es_normalize_rewards(buf.ctypes.data_as(P), buf.size, 1e-8, buf.ctypes.data_as(P))
+    assert st == E.ES_OK
+    assert np.allclose(buf, want, rtol=1e-14, atol=1e-14)
+
+
+def test_assign_index_bases_overflow_returns_zero(E):
+    segs = [E.Segment(0, 2**63), E.Segment(0, 2**63 + 16)]
+    assert E.es_assign_index_bases(segs) == 0
