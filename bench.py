@@ -288,6 +288,10 @@ MUFU_PER_GAUSS = 2
 MUFU_PER_CLK_SM = 16
 
 
+# The device code of the kernels whose DRAM traffic is recorded.
+KERNEL_SOURCES = ("es_internal.h", "es_kernels.cu", "es_noise.cuh")
+
+
 def traffic_per_element(kind):
     """DRAM bytes per parameter of one launch from the committed ncu summary,
     or None if the kernel sources changed since that capture."""
@@ -297,7 +301,7 @@ def traffic_per_element(kind):
         return None
     h = hashlib.sha256()
     csrc = os.path.join(ROOT, "paper_2608_17310_gb300", "csrc")
-    for f in sorted(os.listdir(csrc)):
+    for f in KERNEL_SOURCES:
         with open(os.path.join(csrc, f), "rb") as fh:
             h.update(fh.read())
     digest = h.hexdigest()[:16]
