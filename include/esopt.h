@@ -48,6 +48,10 @@
  *     repeated calls give bit-identical parameters on every run.
  *   - Thread safety: distinct plans may be used from different threads; one plan
  *     must not be used on two streams at once.
+ *   - Plan-based device entry points neither synchronise the host nor allocate
+ *     per call, so they can be recorded in a CUDA graph (stream capture); the
+ *     host arguments of a captured call (seeds, coefficients, sigma) are fixed
+ *     at capture time.
  */
 #ifndef ESOPT_H_
 #define ESOPT_H_

@@ -437,3 +437,37 @@ def test_special_values(es, oracle, dtype):
     tol = noise_abs_tol([oracle.noise_at(9, g)], [0.5])[fin]
     compare(dtype, got[fin], want[fin], f"special values {dtype}", tol)
     plan.close()
+
+
+def test_generation_captured_in_a_cuda_graph_replays_bit_identically(es):
+    # The device entry points make no host synchronisation and allocate
+    # nothing per call, so a generation can be captured once and replayed; the
+    # host-side arguments (seeds, coefficients) are fixed at capture.
+    a = make_params("bf16", [100003, 8192 + 7], seed=17)
+    b = [t.clone() for t in a]
+    plan_a, _ = build_plan(es, a)
+    plan_b, _ = build_plan(es, b)
+    seeds = np.arange(60, 68, dtype=np.uint64)
+    coeffs = np.linspace(-1e-3, 1e-3, 8).astype(np.float32)
+
+    def generation(plan, stream=None):
+        es.es_perturb(plan, int(seeds[0]), 1e-3, stream)
+        for i in range(1, 8):
+            es.es_restore_perturb(plan, int(seeds[i - 1]), 1e-3, int(seeds[i]), 1e-3, stream)
+        es.es_restore(plan, int(seeds[7]), 1e-3, stream)
+        es.es_update(plan, seeds, coeffs, stream)
+
+    for _ in range(3):
+        generation(plan_a)
+    s = torch.cuda.Stream()
+    s.wait_stream(torch.cuda.current_stream())
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g, stream=s):
+        generation(plan_b, s)
+    for _ in range(3):
+        g.replay()
+    torch.cuda.synchronize()
+    for x, y in zip(a, b):
+        assert torch.equal(_int_view(x), _int_view(y))
+    plan_a.close()
+    plan_b.close()
