@@ -471,6 +471,31 @@ class PinnedHostBuffer:
         self.tensor = None
 
 
+def host_memory_available() -> int:
+    """MemAvailable of this node in bytes (0 if unknown)."""
+    try:
+        with open("/proc/meminfo") as f:
+            for line in f:
+                if line.startswith("MemAvailable:"):
+                    return int(line.split()[1]) * 1024
+    except OSError:
+        pass
+    return 0
+
+
+def e2e_fits(torch, nbytes: int, dist) -> bool:
+    """Whether every rank on this node can page-lock its own copy of the
+    parameter set with room to spare; all ranks take the same decision."""
+    local = int(os.environ.get("LOCAL_WORLD_SIZE", "1"))
+    ok = host_memory_available() >= 1.5 * local * nbytes
+    if dist is None:
+        return ok
+    dev = "cuda" if dist.get_backend() == "nccl" else "cpu"
+    t = torch.tensor([1 if ok else 0], dtype=torch.int32, device=dev)
+    dist.all_reduce(t, op=dist.ReduceOp.MIN)
+    return bool(t.item())
+
+
 def run_e2e(args, torch, es, plan, flat, params, wl, n, esize, sigma_at, s_handle, dist, world,
             fused, groups=8, nstreams=4):
     """Same generation with the parameter set in pinned host memory: every step
@@ -480,6 +505,12 @@ def run_e2e(args, torch, es, plan, flat, params, wl, n, esize, sigma_at, s_handl
     its copy back starts when its last pass is done (the middle passes use the
     whole plan). The results are those of the unsplit calls: every call is
     elementwise."""
+    nbytes = flat.numel() * esize
+    if not e2e_fits(torch, nbytes, dist):
+        local = int(os.environ.get("LOCAL_WORLD_SIZE", "1"))
+        return {"value": None, "unit": UNIT, "unavailable":
+                f"host memory: {local} ranks x {nbytes / 1e9:.1f} GB page-locked would exceed "
+                f"2/3 of the {host_memory_available() / 1e9:.0f} GB available"}
     pinned = PinnedHostBuffer(torch, flat)
     host = pinned.tensor
     host.copy_(flat)
