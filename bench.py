@@ -292,19 +292,53 @@ MUFU_PER_CLK_SM = 16
 KERNEL_SOURCES = ("es_internal.h", "es_kernels.cu", "es_noise.cuh")
 
 
+def strip_comments(src):
+    """C/C++ source without comments, trailing blanks or blank lines, so that
+    an edit to comments or layout leaves the code digest unchanged. String and
+    character literals are kept as written."""
+    out, i, n = [], 0, len(src)
+    while i < n:
+        c = src[i]
+        if src.startswith("//", i):
+            j = src.find("\n", i)
+            i = n if j < 0 else j
+        elif src.startswith("/*", i):
+            j = src.find("*/", i + 2)
+            i = n if j < 0 else j + 2
+            out.append(" ")
+        elif c in "\"'":
+            j = i + 1
+            while j < n and src[j] != c:
+                j += 2 if src[j] == "\\" else 1
+            out.append(src[i:j + 1])
+            i = j + 1
+        else:
+            out.append(c)
+            i += 1
+    lines = (" ".join(line.split()) for line in "".join(out).split("\n"))
+    return "\n".join(line for line in lines if line)
+
+
+def kernel_code_digest(csrc=None):
+    """First 16 hex digits of the sha256 over the kernels' device sources
+    (KERNEL_SOURCES in order), comments and layout stripped."""
+    import hashlib
+    csrc = csrc or os.path.join(ROOT, "paper_2608_17310_gb300", "csrc")
+    h = hashlib.sha256()
+    for f in KERNEL_SOURCES:
+        with open(os.path.join(csrc, f), encoding="utf-8") as fh:
+            h.update(strip_comments(fh.read()).encode())
+            h.update(b"\0")
+    return h.hexdigest()[:16]
+
+
 def traffic_per_element(kind):
     """DRAM bytes per parameter of one launch from the committed ncu summary,
-    or None if the kernel sources changed since that capture."""
-    import hashlib
+    or None if the kernels' code changed since that capture."""
     path = os.path.join(ROOT, "profiles", "dram_traffic.txt")
     if not os.path.exists(path):
         return None
-    h = hashlib.sha256()
-    csrc = os.path.join(ROOT, "paper_2608_17310_gb300", "csrc")
-    for f in KERNEL_SOURCES:
-        with open(os.path.join(csrc, f), "rb") as fh:
-            h.update(fh.read())
-    digest = h.hexdigest()[:16]
+    digest = kernel_code_digest()
     for line in open(path):
         f = line.split()
         if len(f) == 3 and not line.startswith("#") and f[0] == kind:

@@ -2,7 +2,7 @@
  * esopt.h -- C ABI of the GB300 (sm_103a) library for the parameter-space
  * evolution-strategies (ES) step of Agentic ESOpt.
  *
- * One ES generation as the paper states it (§3 "Methodology", §3.1, App. D.6):
+ * One ES generation as the paper states it (§3, §3.1, App. D.6):
  *
  *   sigma_t = cosine schedule (§3.1)                       es_sigma_cosine
  *   for each member i with integer seed s_i:
@@ -14,8 +14,9 @@
  *   theta <- theta + sum_i c_i * eps_{s_i}    (one pass)    es_update
  *
  * The noise eps_s is never stored: it is regenerated from the seed whenever it
- * is needed ("storing only the noise seed", §3; App. D.6). The paper does not
- * name a generator; this library fixes it as follows, for every entry point:
+ * is needed: per member only its integer seed is kept (§3; App. D.6). The
+ * paper does not name a generator; this library fixes it as follows, for every
+ * entry point:
  *
  *   block j = floor(g / 4) of global parameter index g,
  *   Philox4x32-10 (Salmon et al., SC'11) with key = (seed_lo32, seed_hi32) and
@@ -94,8 +95,8 @@ typedef enum {
 } es_scale_t;
 
 /*
- * One parameter tensor of the full parameter set ("full-parameter"
- * perturbation covers every tensor, §3 and App. D.6).
+ * One parameter tensor of the full parameter set (the perturbation reaches
+ * every tensor of the model, §3 and App. D.6).
  *   data        device pointer to `numel` contiguous elements of the plan's
  *               dtype; must be 16-byte aligned; owned by the caller and must
  *               stay valid while the plan is used.
@@ -114,8 +115,11 @@ typedef struct es_plan* es_plan_t;
 
 /*
  * Validates the segment list and copies it to the current device (one
- * cudaMalloc of about 32 bytes per segment; synchronous). The segment list
- * itself may be freed after the call. The plan is immutable.
+ * cudaMalloc of about 32 bytes per segment; synchronous). Every segment must
+ * lie in device (or managed) memory of the current device: host pointers,
+ * page-locked or not, are rejected with ES_ERR_INVALID_ARG, since a kernel
+ * given one could fault. The segment list itself may
+ * be freed after the call. The plan is immutable.
  * Errors: ES_ERR_INVALID_ARG (segs or out NULL, nseg < 1, numel 0, bad dtype,
  * index range past 2^64), ES_ERR_ALIGNMENT, ES_ERR_OVERLAP,
  * ES_ERR_NO_MEMORY, ES_ERR_CUDA. On error *out is set to NULL.
@@ -139,10 +143,10 @@ uint64_t es_assign_index_bases(es_segment_t* segs, int nseg);
 
 /*
  * out[k] = eps_seed[index_base + k] for k in [0, n), as fp32 on the device.
- * Any index_base and n (n = 0 is a no-op); `out` must be 4-byte aligned and
- * index_base + n must not pass 2^64. Regenerates exactly the values the other
- * device entry points use (App. D.6: "reconstructs the same direction from its
- * integer seed").
+ * Any index_base and n (n = 0 is a no-op); `out` must be device memory of the
+ * current device, 4-byte aligned, and index_base + n must not pass 2^64.
+ * Regenerates exactly the values the other device entry points use: the update
+ * rebuilds each member's direction from its seed alone (App. D.6).
  */
 es_status_t es_noise_fill(uint64_t seed, uint64_t index_base, uint64_t n,
                           float* out, void* stream);
@@ -152,9 +156,10 @@ es_status_t es_noise_fill(uint64_t seed, uint64_t index_base, uint64_t n,
  * out[4t + w] = word w (0..3) of Philox4x32-10 block (block_base + t) of
  * `seed`, for t in [0, nblocks); block j holds the noise of global indices
  * 4j .. 4j+3. For checking the integer stream bit for bit (reproducibility
- * across runs, devices and implementations). `out` is a device buffer of
- * 4 * nblocks words and must be 16-byte aligned; nblocks = 0 is a no-op and
- * block_base + nblocks must not pass 2^62.
+ * across runs, devices and implementations). `out` is a buffer of
+ * 4 * nblocks words in device memory of the current device and must be
+ * 16-byte aligned; nblocks = 0 is a no-op and block_base + nblocks must not
+ * pass 2^62.
  * Errors: ES_ERR_INVALID_ARG, ES_ERR_ALIGNMENT, ES_ERR_CUDA.
  */
 es_status_t es_noise_bits(uint64_t seed, uint64_t block_base, uint64_t nblocks,
@@ -167,14 +172,16 @@ es_status_t es_noise_bits(uint64_t seed, uint64_t block_base, uint64_t nblocks,
  *   out[2k]   = r cos(2 pi u(words[2k+1])),  out[2k+1] = r sin(2 pi u(words[2k+1])),
  *   r = sqrt(-2 ln u(words[2k])),  u(x) = (2 (x >> 9) + 1) / 2^24.
  * Each word matters only through its top 23 bits, so this lets the transform
- * be checked over its whole input domain. `words` and `out` are device
- * buffers of 2 * npairs entries, 8-byte aligned; npairs = 0 is a no-op.
+ * be checked over its whole input domain. `words` and `out` are buffers of
+ * 2 * npairs entries in device memory of the current device, 8-byte aligned;
+ * npairs = 0 is a no-op.
  * Errors: ES_ERR_INVALID_ARG, ES_ERR_ALIGNMENT, ES_ERR_CUDA.
  */
 es_status_t es_box_muller(const uint32_t* words, uint64_t npairs, float* out, void* stream);
 
 /*
- * Perturb in place (§3; App. D.6 "applies theta + sigma_t eps_i"):
+ * Perturb in place, theta + sigma_t eps_i before member i's rollout (§3;
+ * App. D.6):
  * theta[g] <- round(theta[g] + sigma * eps_seed[g]) for every element of every
  * segment, with the product and sum in fp32 (one fused multiply-add) and one
  * rounding to the storage type (round to nearest even).
@@ -184,8 +191,8 @@ es_status_t es_box_muller(const uint32_t* words, uint64_t npairs, float* out, vo
 es_status_t es_perturb(es_plan_t plan, uint64_t seed, float sigma, void* stream);
 
 /*
- * Restore in place after the rollout (§3 "in-place addition and subtraction";
- * App. D.6 "reverts the perturbation"):
+ * Restore in place after the rollout: the perturbation is subtracted from the
+ * same buffer it was added to (§3; App. D.6):
  * theta[g] <- round(theta[g] - sigma * eps_seed[g]), same seed and sigma as the
  * es_perturb it undoes. In fp32 storage the round trip returns theta to within
  * one rounding; in bf16 an element can end one ulp away where theta + sigma*eps
@@ -218,7 +225,8 @@ es_status_t es_restore_perturb(es_plan_t plan, uint64_t restore_seed, float sigm
  * type, so theta is read and written exactly once. `seeds` and `coeffs` are
  * host arrays of length n (1 <= n <= ES_MAX_SEEDS). Seeds whose coefficient is
  * 0 are skipped; if every coefficient is 0 nothing is launched and theta stays
- * bit-identical ("an all-invalid batch produces no update", App. D.5/D.6).
+ * bit-identical (a batch with no valid reward leaves theta unchanged,
+ * App. D.5/D.6).
  * Errors: ES_ERR_INVALID_ARG, ES_ERR_TOO_MANY_SEEDS, ES_ERR_NONFINITE,
  * ES_ERR_WRONG_DEVICE, ES_ERR_CUDA.
  */
@@ -261,8 +269,8 @@ es_status_t es_replay(es_plan_t plan, const uint64_t* seeds, const float* coeffs
  * Population z-score of the rewards (§3):
  *   rhat_i = (R_i - mu) / (s + eps_z),  mu = (1/G) sum R_j,
  *   s^2 = (1/G) sum (R_j - mu)^2  (population variance).
- * Non-finite rewards first receive a finite within-batch penalty, the smallest
- * finite reward of the batch (the rule for invalid candidates of §5 and
+ * A non-finite reward is first replaced by a finite penalty taken from the
+ * batch itself, its smallest finite reward (the rule for invalid candidates of §5 and
  * App. D.5/D.6). If no reward is finite, or all are equal, every rhat_i is 0
  * (no update). Host-only. `rewards` and `rhat` may alias.
  * Errors: ES_ERR_INVALID_ARG (NULL, n < 1, eps_z < 0 or not finite).
@@ -271,7 +279,7 @@ es_status_t es_normalize_rewards(const double* rewards, int n, double eps_z,
                                  double* rhat);
 
 /*
- * Cosine decay of the perturbation radius (§3.1):
+ * Cosine schedule of sigma over the T generations (§3.1):
  *   sigma_t = sigma_T + (sigma_0 - sigma_T) (1 + cos(pi t / T)) / 2,
  * t clamped to [0, T]. Generation t = 0..T-1 uses sigma_t, so sigma_0 is used
  * first and sigma_T is the value after the last generation. T <= 0 returns
@@ -312,8 +320,9 @@ es_status_t es_fold_antithetic(const double* rhat_pos, const double* rhat_neg,
  *
  * theta[g] <- round(theta[g] + sigma * eps_seed[g]) over the given segments,
  * exactly as es_perturb on a plan made from the same segments; pass -sigma to
- * restore. Segments follow the rules of es_plan_create (16-byte aligned data,
- * index bases multiples of 8, no overlap) and are validated on every call.
+ * restore. Segments follow the rules of es_plan_create (device memory of the
+ * current device, 16-byte aligned data, index bases multiples of 8, no
+ * overlap) and are validated on every call.
  *
  * Instead of a plan's table, the segment table is copied (cudaMemcpyAsync on
  * `stream`) into one static device array of ES_STATIC_MAX_SEGMENTS + 1

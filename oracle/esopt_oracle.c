@@ -245,8 +245,8 @@ void oracle_update_bf16(uint16_t* theta, const uint64_t* g, uint64_t n,
  * mu = (1/G) sum R_j and s^2 = (1/G) sum (R_j - mu)^2.
  *
  * Invalid rewards (§5 and App. D.5/D.6, automatic heuristic design): a
- * non-finite reward receives a finite within-batch penalty before
- * normalisation; this oracle uses the smallest finite reward of the batch.
+ * non-finite reward is replaced, before normalisation, by a finite penalty
+ * drawn from the same batch; this oracle uses its smallest finite reward.
  * A batch with no finite reward, or whose rewards are all equal, produces no
  * update: every Rhat_i is 0.
  *
@@ -284,7 +284,7 @@ int oracle_zscore(const double* R, int n, double eps_z, double* Rhat) {
 }
 
 /*
- * Cosine decay of the perturbation radius (§3.1):
+ * Cosine schedule of sigma over the T generations (§3.1):
  * sigma_t = sigma_T + (sigma_0 - sigma_T) (1 + cos(pi t / T)) / 2, t = 0..T.
  * t is clamped to [0, T]; T <= 0 gives sigma_0.
  */

@@ -13,6 +13,7 @@
 
 #include "../../include/esopt.h"
 #include "es_internal.h"
+#include "es_memcheck.h"
 #include "es_noise.cuh"
 
 struct es_plan {
@@ -54,6 +55,16 @@ es_status_t check_plan_device(const es_plan* plan) {
   if (cur != plan->device)
     return fail(ES_ERR_WRONG_DEVICE, "plan lives on device %d but device %d is current",
                 plan->device, cur);
+  return ES_OK;
+}
+
+es_status_t check_device_buffer(const void* p, const char* what) {
+  int device = -1;
+  cudaError_t err = cudaGetDevice(&device);
+  if (err != cudaSuccess) return cuda_fail(err, "cudaGetDevice");
+  if (!esopt::is_device_memory(p, device))
+    return fail(ES_ERR_INVALID_ARG, "%s: buffer is not device memory of the current device %d",
+                what, device);
   return ES_OK;
 }
 
@@ -195,13 +206,16 @@ es_status_t es_plan_create(const es_segment_t* segs, int nseg, es_dtype_t dtype,
   }
   table[nseg] = esopt::SegDesc{nullptr, 0, 0, tiles};
 
+  int device = -1;
+  cudaError_t err = cudaGetDevice(&device);
+  if (err != cudaSuccess) return cuda_fail(err, "cudaGetDevice");
+  for (int k = 0; k < nseg; ++k)
+    if (!esopt::is_device_memory(segs[k].data, device))
+      return fail(ES_ERR_INVALID_ARG, "segment %d: not device memory of the current device %d",
+                  k, device);
   es_plan* plan = new (std::nothrow) es_plan{};
   if (plan == nullptr) return fail(ES_ERR_NO_MEMORY, "es_plan_create: host allocation failed");
-  cudaError_t err = cudaGetDevice(&plan->device);
-  if (err != cudaSuccess) {
-    delete plan;
-    return cuda_fail(err, "cudaGetDevice");
-  }
+  plan->device = device;
   const size_t bytes = table.size() * sizeof(esopt::SegDesc);
   err = cudaMalloc(reinterpret_cast<void**>(&plan->d_segs), bytes);
   if (err != cudaSuccess) {
@@ -258,6 +272,8 @@ es_status_t es_noise_fill(uint64_t seed, uint64_t index_base, uint64_t n, float*
     return fail(ES_ERR_ALIGNMENT, "es_noise_fill: out is not 4-byte aligned");
   if (index_base > UINT64_MAX - n)
     return fail(ES_ERR_INVALID_ARG, "es_noise_fill: index range passes 2^64");
+  es_status_t st = check_device_buffer(out, "es_noise_fill");
+  if (st != ES_OK) return st;
   cudaError_t err = esopt::launch_noise_fill(seed, index_base, n, out,
                                              static_cast<cudaStream_t>(stream));
   if (err != cudaSuccess) return cuda_fail(err, "es_noise_fill");
@@ -273,6 +289,8 @@ es_status_t es_noise_bits(uint64_t seed, uint64_t block_base, uint64_t nblocks, 
   const uint64_t kMaxBlock = uint64_t{1} << 62;
   if (block_base > kMaxBlock || nblocks > kMaxBlock - block_base)
     return fail(ES_ERR_INVALID_ARG, "es_noise_bits: block range passes 2^62");
+  es_status_t st = check_device_buffer(out, "es_noise_bits");
+  if (st != ES_OK) return st;
   cudaError_t err = esopt::launch_noise_bits(seed, block_base, nblocks, out,
                                              static_cast<cudaStream_t>(stream));
   if (err != cudaSuccess) return cuda_fail(err, "es_noise_bits");
@@ -287,6 +305,9 @@ es_status_t es_box_muller(const uint32_t* words, uint64_t npairs, float* out, vo
     return fail(ES_ERR_ALIGNMENT, "es_box_muller: buffers must be 8-byte aligned");
   if (npairs > (UINT64_MAX >> 4))
     return fail(ES_ERR_INVALID_ARG, "es_box_muller: npairs too large");
+  es_status_t st = check_device_buffer(words, "es_box_muller");
+  if (st == ES_OK) st = check_device_buffer(out, "es_box_muller");
+  if (st != ES_OK) return st;
   cudaError_t err = esopt::launch_box_muller(words, npairs, out, static_cast<cudaStream_t>(stream));
   if (err != cudaSuccess) return cuda_fail(err, "es_box_muller");
   return ok();

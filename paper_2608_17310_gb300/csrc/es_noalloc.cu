@@ -13,6 +13,7 @@
 
 #include "../../include/esopt.h"
 #include "es_internal.h"
+#include "es_memcheck.h"
 
 namespace esopt {
 namespace {
@@ -115,6 +116,10 @@ extern "C" es_status_t es_perturb_noalloc(const es_segment_t* segs, int nseg, es
   if (device < 0 || device >= esopt::kMaxDevices)
     return reject(ES_ERR_INVALID_ARG, "es_perturb_noalloc: device ordinal %d >= %d", device,
                   esopt::kMaxDevices);
+  for (int k = 0; k < nseg; ++k)
+    if (!esopt::is_device_memory(segs[k].data, device))
+      return reject(ES_ERR_INVALID_ARG,
+                    "es_perturb_noalloc: segment %d is not device memory of device %d", k, device);
   SegDesc* d_table = nullptr;
   es_status_t st = esopt::table_address(device, &d_table);
   if (st != ES_OK) return st;

@@ -1,7 +1,7 @@
 // Counter-based Gaussian noise for the ES step, regenerated from the integer
 // seed wherever it is needed (§3: only the seed of each perturbation is
-// stored; App. D.6: the update "reconstructs the same direction from its
-// integer seed").
+// stored; App. D.6: the update rebuilds each member's direction from that
+// seed alone).
 //
 // Definition (fixed by this library; the paper names no generator):
 //   block j = floor(g / 4) of global parameter index g;

@@ -209,6 +209,8 @@ def segments_from_tensors(tensors, index_bases=None):
     """Segments for a list of contiguous CUDA tensors (bases assigned if None)."""
     segs = []
     for t in tensors:
+        if not t.is_cuda:
+            raise ValueError("parameter tensors must be CUDA tensors")
         if not t.is_contiguous():
             raise ValueError("parameter tensors must be contiguous")
         segs.append(Segment(int(t.data_ptr()), int(t.numel()), 0))

@@ -1,0 +1,42 @@
+"""Host logic of bench.py that needs no GPU: the code digest that decides
+whether the committed DRAM traffic still describes the kernels."""
+import os
+import shutil
+
+import bench
+
+CSRC = os.path.join(bench.ROOT, "paper_2608_17310_gb300", "csrc")
+
+
+def test_strip_comments_keeps_literals_and_drops_comments():
+    src = 'a = "x // y /* z */"; // gone\n/* gone\n too */ b = \'/\';  \n\n  c  =  1;\n'
+    assert bench.strip_comments(src) == 'a = "x // y /* z */";\nb = \'/\';\nc = 1;'
+    assert bench.strip_comments('asm("mov.b32 %0, %1;" : "=r"(x));') == \
+        'asm("mov.b32 %0, %1;" : "=r"(x));'
+
+
+def _copy_sources(tmp_path):
+    for f in bench.KERNEL_SOURCES:
+        shutil.copy(os.path.join(CSRC, f), tmp_path / f)
+    return str(tmp_path)
+
+
+def test_comment_edit_keeps_the_digest_and_code_edit_changes_it(tmp_path):
+    d = _copy_sources(tmp_path)
+    base = bench.kernel_code_digest(d)
+    assert base == bench.kernel_code_digest(CSRC)
+    p = tmp_path / "es_noise.cuh"
+    text = p.read_text()
+    p.write_text("// a new comment line\n" + text.replace("\n", "   \n", 3) + "\n/* tail */\n")
+    assert bench.kernel_code_digest(d) == base
+    p.write_text(text.replace("0xD2511F53u", "0xD2511F55u"))
+    assert bench.kernel_code_digest(d) != base
+
+
+def test_traffic_file_is_keyed_by_a_well_formed_digest():
+    rows = [line.split() for line in open(os.path.join(bench.ROOT, "profiles", "dram_traffic.txt"))
+            if line.strip() and not line.startswith("#")]
+    assert {r[0] for r in rows} == {"restore_perturb", "update_perturb"}
+    for kind, per_param, digest in rows:
+        assert 2.0 < float(per_param) < 8.0
+        assert len(digest) == 16 and int(digest, 16) >= 0

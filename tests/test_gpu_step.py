@@ -471,3 +471,24 @@ def test_generation_captured_in_a_cuda_graph_replays_bit_identically(es):
         assert torch.equal(_int_view(x), _int_view(y))
     plan_a.close()
     plan_b.close()
+
+
+def test_host_buffers_are_refused_before_any_launch(es):
+    # Page-locked host tensors: device-accessible through unified addressing,
+    # so nothing could fault even if a launch happened; the library must still
+    # refuse them (parameters belong in device memory) and leave them untouched.
+    host = torch.zeros(4096, dtype=torch.float32).pin_memory()
+    bits = torch.zeros(64, dtype=torch.int32).pin_memory()
+    seg = [es.Segment(int(host.data_ptr()), host.numel(), 0)]
+    for call in (lambda: es.es_plan_create(seg, es.ES_FP32),
+                 lambda: es.es_perturb_noalloc(seg, es.ES_FP32, 1, 1e-3),
+                 lambda: es.es_noise_fill(1, 0, host.numel(), host),
+                 lambda: es.es_noise_bits(1, 0, 16, bits)):
+        with pytest.raises(es.EsError) as err:
+            call()
+        assert err.value.status == es.ES_ERR_INVALID_ARG
+        assert "not device memory" in es.es_last_error()
+    torch.cuda.synchronize()
+    assert not host.any() and not bits.any()
+    with pytest.raises(ValueError):
+        es.plan_from_tensors([host])
