@@ -4,6 +4,7 @@ synthetic parameter set shaped like the paper's workloads.
 
     python bench.py [--gpus N] [--steps K] [--warmup W] [--workload qwen27b]
                     [--impl ours|reference] [--no-e2e] [--no-cpu-baseline]
+    python bench.py --sweep [--populations 1,2,4,...] [--workload qwen4b]
 
 Prints one JSON line (rank 0). `value` is measured with the inputs resident in
 HBM; `e2e` is the same metric with the parameters in pinned host memory and
@@ -52,7 +53,15 @@ def parse():
     p.add_argument("--e2e-steps", type=int, default=2)
     p.add_argument("--unfused", action="store_true",
                    help="separate es_restore / es_perturb launches instead of es_restore_perturb")
-    return p.parse_args()
+    p.add_argument("--sweep", action="store_true",
+                   help="instead of the step: time es_update alone for each N of --populations "
+                        "(default workload qwen4b) and print one JSON line with every point")
+    p.add_argument("--populations", default="1,2,4,8,16,32,64,128",
+                   help="comma-separated N values of --sweep")
+    args = p.parse_args()
+    if args.sweep and "--workload" not in " ".join(sys.argv):
+        args.workload = "qwen4b"
+    return args
 
 
 def peaks():
@@ -395,12 +404,7 @@ def run_ours(args, rank, world, dist):
     per_step_ms = ms_max / args.steps
     value = world * P * n * args.steps / (ms_max / 1e3)
 
-    hbm_gbs, sm_max_mhz, peak_src = peaks()
-    sms = torch.cuda.get_device_properties(dev_index).multi_processor_count
-    imul_peak = sms * IMUL_PER_CLK_SM * sm_max_mhz * 1e6          # 32-bit multiplies / s
-    gauss_peak = imul_peak / IMUL_PER_GAUSS
-    shared_peak = sms * sm_max_mhz * 1e6 / (IMUL_PER_GAUSS / IMUL_PER_CLK_SM +
-                                             MUFU_PER_GAUSS / MUFU_PER_CLK_SM)
+    imul_peak, gauss_peak, shared_peak, sms, sm_max_mhz, hbm_gbs, peak_src = alu_peaks(torch, dev_index)
     bytes_per_launch = 2 * esize * P
     kernels = {}
     for name in timers.names():
@@ -462,6 +466,92 @@ def run_ours(args, rank, world, dist):
         "cpu_baseline": cpu,
     }
     plan.close()
+    if rank == 0:
+        print(json.dumps(out), flush=True)
+
+
+def alu_peaks(torch, dev_index):
+    """(imul32/s, Gaussians/s at the integer-multiply roofline, Gaussians/s at
+    the IMUL+MUFU bound, SM count, max SM MHz, HBM GB/s, peak source)."""
+    hbm_gbs, sm_max_mhz, peak_src = peaks()
+    sms = torch.cuda.get_device_properties(dev_index).multi_processor_count
+    imul_peak = sms * IMUL_PER_CLK_SM * sm_max_mhz * 1e6
+    shared_peak = sms * sm_max_mhz * 1e6 / (IMUL_PER_GAUSS / IMUL_PER_CLK_SM +
+                                             MUFU_PER_GAUSS / MUFU_PER_CLK_SM)
+    return imul_peak, imul_peak / IMUL_PER_GAUSS, shared_peak, sms, sm_max_mhz, hbm_gbs, peak_src
+
+
+def run_sweep(args, rank, world, dist):
+    """es_update alone on one parameter set for each population size N: where
+    the fused update turns from HBM-bound (small N: 2 * sizeof bytes per
+    parameter, N Gaussians) to generator-bound (large N). Each launch is timed
+    with CUDA events on the launching stream; the set is larger than L2."""
+    import torch
+    from paper_2608_17310_gb300 import build, esopt as es
+
+    build.build_library()
+    dev_index = torch.cuda.current_device()
+    torch.cuda.init()
+    wl = I.WORKLOADS[args.workload]
+    specs = I.shapes_for(args.workload)
+    dtype = torch.bfloat16 if wl.dtype == "bf16" else torch.float32
+    esize = 2 if wl.dtype == "bf16" else 4
+    flat, params = I.init_params_flat(specs, dtype, "cuda", seed=0)
+    plan = es.plan_from_tensors(params)
+    P = plan.numel
+    stream = torch.cuda.current_stream()
+    s_handle = stream.cuda_stream
+    imul_peak, gauss_peak, shared_peak, sms, sm_max_mhz, hbm_gbs, peak_src = alu_peaks(torch, dev_index)
+    bytes_per_launch = 2 * esize * P
+    pops = [int(x) for x in args.populations.split(",") if x.strip()]
+    points = []
+    launches = 0
+    with ClockSampler(dev_index) as clk:
+        for n in pops:
+            seeds = I.population_seeds(n, generation=n, first=7)
+            # N(0, 1) rewards used as the normalised rewards directly (a z-score
+            # of a single reward would be 0: no update to time at N = 1)
+            rhat = I.rewards("normal", n, seed=n)
+            coeffs = es.es_update_coeffs(rhat, wl.alpha, float(np.float32(wl.sigma)),
+                                         es.ES_SCALE_PAPER)
+            for _ in range(args.warmup):
+                es.es_update(plan, seeds, coeffs, s_handle)
+            torch.cuda.synchronize()
+            evs = []
+            for _ in range(args.steps):
+                e0 = torch.cuda.Event(enable_timing=True)
+                e1 = torch.cuda.Event(enable_timing=True)
+                e0.record(stream)
+                es.es_update(plan, seeds, coeffs, s_handle)
+                e1.record(stream)
+                evs.append((e0, e1))
+                launches += 1
+            torch.cuda.synchronize()
+            ms = sum(a.elapsed_time(b) for a, b in evs) / len(evs) if evs else float("nan")
+            gbs = bytes_per_launch / (ms / 1e3) / 1e9
+            gps = n * P / (ms / 1e3)
+            t_hbm = bytes_per_launch / (hbm_gbs * 1e9) * 1e3
+            t_imul = n * P / gauss_peak * 1e3
+            t_shared = n * P / shared_peak * 1e3
+            points.append({
+                "population": n, "mean_ms": ms, "gbs": gbs, "gauss_per_s": gps,
+                "hbm_frac": gbs / hbm_gbs, "alu_frac": gps / gauss_peak,
+                "imul_mufu_frac": gps / shared_peak,
+                "bound": "alu" if t_imul > t_hbm else "hbm",
+                "roofline_frac": max(t_hbm, t_imul) / ms,
+                "t_hbm_ms": t_hbm, "t_imul_ms": t_imul, "t_imul_mufu_ms": t_shared})
+    plan.close()
+    out = {"mode": "sweep", "metric": "es_update param*seed/s per population size",
+           "unit": UNIT, "n_gpus": 1, "steps": args.steps, "warmup": args.warmup,
+           "dtype": "f32", "data": "synthetic",
+           "config": dict(workload_config(args.workload, pops[-1] if pops else 0, 1),
+                          populations=pops, call="es_update",
+                          rewards="N(0,1) used as the normalised rewards; paper-scale coefficients"),
+           "peaks": {"hbm_gbs": hbm_gbs, "hbm_source": peak_src,
+                     "imul32_per_s": imul_peak, "gauss_per_s_imul": gauss_peak,
+                     "gauss_per_s_imul_mufu": shared_peak, "sms": sms, "sm_max_mhz": sm_max_mhz},
+           "bytes_per_launch": bytes_per_launch, "points": points,
+           "gpu_launches": launches, "clocks": clk.summary()}
     if rank == 0:
         print(json.dumps(out), flush=True)
 
@@ -713,6 +803,8 @@ def main():
     try:
         if args.impl == "reference":
             run_reference(args, rank, world, dist)
+        elif args.sweep:
+            run_sweep(args, rank, world, dist)
         else:
             run_ours(args, rank, world, dist)
     finally:
