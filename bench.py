@@ -768,7 +768,7 @@ def cpu_baseline(workload, n, sigma, sample=CPU_SAMPLE):
                       f"{secs:.1f} s"}
 
 
-def run_reference(args, rank, world, dist):
+def run_reference(args, rank, world):
     if rank != 0:
         return
     wl = I.WORKLOADS[args.workload]
@@ -799,11 +799,14 @@ def run_reference(args, rank, world, dist):
 
 def main():
     args = parse()
+    if args.impl == "reference":
+        # CPU work on rank 0 alone: no process group and no GPU for any rank.
+        run_reference(args, int(os.environ.get("RANK", "0")),
+                      int(os.environ.get("WORLD_SIZE", "1")))
+        return
     rank, world, dist = dist_setup(args)
     try:
-        if args.impl == "reference":
-            run_reference(args, rank, world, dist)
-        elif args.sweep:
+        if args.sweep:
             run_sweep(args, rank, world, dist)
         else:
             run_ours(args, rank, world, dist)

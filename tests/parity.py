@@ -61,3 +61,30 @@ def assert_bf16_within_ulp(got_bits, want_bits, what="", ulps=1, abs_tol=0.0):
     assert bad.size == 0, (f"{what}: {bad.size} of {d.size} bf16 values more than {ulps} ulp "
                            f"apart; first at {bad[:5]}: got {np.asarray(got_bits)[bad[:5]]} "
                            f"want {np.asarray(want_bits)[bad[:5]]}")
+
+
+def build_c_consumer(out_dir):
+    """Compiles tests/abi_c_consumer.c (C99) against include/esopt.h and links
+    it to the in-tree libesopt.so and the CUDA runtime. Returns the path of
+    the executable."""
+    import glob
+    import os
+    import subprocess
+    here = os.path.dirname(os.path.abspath(__file__))
+    root = os.path.dirname(here)
+    cuda = os.environ.get("CUDA_HOME", "/usr/local/cuda")
+    libdirs = [d for d in [os.path.join(cuda, "lib64")] + glob.glob(os.path.join(cuda, "targets", "*", "lib"))
+               if glob.glob(os.path.join(d, "libcudart.so*"))]
+    if not libdirs:
+        raise RuntimeError("libcudart.so not found under " + cuda)
+    build = os.path.join(root, "paper_2608_17310_gb300", "_build")
+    exe = os.path.join(str(out_dir), "abi_c_consumer")
+    cmd = ["gcc", "-std=c99", "-Wall", "-Wextra", "-Werror",
+           f"-I{os.path.join(root, 'include')}", f"-I{os.path.join(cuda, 'include')}",
+           os.path.join(here, "abi_c_consumer.c"), "-o", exe,
+           f"-L{build}", "-lesopt", f"-L{libdirs[0]}", "-lcudart",
+           f"-Wl,-rpath,{build}", f"-Wl,-rpath,{libdirs[0]}"]
+    r = subprocess.run(cmd, capture_output=True, text=True)
+    if r.returncode != 0:
+        raise RuntimeError("building the C consumer failed:\n" + r.stderr)
+    return exe

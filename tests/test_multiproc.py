@@ -18,8 +18,9 @@ def _free_port():
 
 
 def _worker(rank, world, port, q):
+    # CPU ranks on gloo whatever the machine has: GPUs are hidden before torch loads.
     os.environ.update(MASTER_ADDR="127.0.0.1", MASTER_PORT=str(port), RANK=str(rank),
-                      WORLD_SIZE=str(world), LOCAL_RANK=str(rank))
+                      WORLD_SIZE=str(world), LOCAL_RANK=str(rank), CUDA_VISIBLE_DEVICES="")
     sys.path.insert(0, ROOT)
     import bench
     r, w, dist = bench.dist_setup(None)
