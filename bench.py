@@ -355,6 +355,23 @@ def traffic_per_element(kind):
     return None
 
 
+def pipe_occupancy(kind):
+    """FMA-heavy and XU cycles active (% of elapsed) of a launch kind from the
+    committed ncu summary, or None if the kernels' code changed since."""
+    path = os.path.join(ROOT, "profiles", "pipe_occupancy.txt")
+    if not os.path.exists(path):
+        return None
+    digest = kernel_code_digest()
+    for line in open(path):
+        f = line.split()
+        if len(f) == 4 and not line.startswith("#") and f[0] == kind and f[3] == digest:
+            heavy, xu = float(f[1]), float(f[2])
+            return {"fmaheavy_pct": heavy, "xu_pct": xu, "sum_pct": round(heavy + xu, 1),
+                    "source": "ncu sm__pipe_fmaheavy_cycles_active + sm__pipe_xu_cycles_active, "
+                              "profiles/pipe_occupancy.txt"}
+    return None
+
+
 def run_ours(args, rank, world, dist):
     import torch
     from paper_2608_17310_gb300 import build, esopt as es
@@ -437,6 +454,7 @@ def run_ours(args, rank, world, dist):
         "source": f"integer-multiply and MUFU work issue from the same SM sub-partition "
                   f"without overlap: {IMUL_PER_GAUSS}/{IMUL_PER_CLK_SM} + "
                   f"{MUFU_PER_GAUSS}/{MUFU_PER_CLK_SM} SM-clocks per Gaussian"}
+    roof["pipe_occupancy"] = pipe_occupancy(dom)
     roof.update({"kernel": d["kernel"], "hbm_frac": d["hbm_frac"], "alu_frac": d["alu_frac"],
                  "algorithmic_bytes_per_launch": bytes_per_launch,
                  "gaussians_per_launch": gauss_per_elem(dom, n) * P})

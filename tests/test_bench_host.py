@@ -40,3 +40,13 @@ def test_traffic_file_is_keyed_by_a_well_formed_digest():
     for kind, per_param, digest in rows:
         assert 2.0 < float(per_param) < 8.0
         assert len(digest) == 16 and int(digest, 16) >= 0
+
+
+def test_pipe_occupancy_file_is_keyed_by_the_current_code():
+    occ = bench.pipe_occupancy("restore_perturb")
+    rows = [line.split() for line in open(os.path.join(bench.ROOT, "profiles", "pipe_occupancy.txt"))
+            if line.strip() and not line.startswith("#")]
+    assert {r[0] for r in rows} == {"restore_perturb", "update_perturb", "update"}
+    if all(r[3] == bench.kernel_code_digest() for r in rows):
+        assert occ is not None and 90.0 < occ["sum_pct"] < 105.0
+    assert bench.pipe_occupancy("restore") is None
