@@ -492,3 +492,62 @@ def test_host_buffers_are_refused_before_any_launch(es):
     assert not host.any() and not bits.any()
     with pytest.raises(ValueError):
         es.plan_from_tensors([host])
+
+
+@pytest.mark.parametrize("dtype", ["bf16", "f32"])
+def test_zero_sigma_moves_only_the_sign_of_negative_zeros(es, oracle, dtype):
+    # theta + 0 * eps: finite non-zero values, infinities and NaN stay as they
+    # are; -0 becomes the IEEE sum -0 + (0 * eps), whose sign follows eps, and
+    # the oracle takes the same decision in double.
+    rng = np.random.default_rng(12)
+    vals = np.concatenate([0.02 * rng.standard_normal(8192 + 37), [0.0, -0.0] * 64,
+                           [np.inf, -np.inf, np.nan] * 8]).astype(np.float32)
+    t = torch.from_numpy(vals.copy())
+    t = (t.to(torch.bfloat16) if dtype == "bf16" else t).cuda()
+    plan, segs = build_plan(es, [t])
+    g = indices(segs)[0]
+    for call, oracle_call in ((es.es_perturb, oracle.perturb), (es.es_restore, oracle.restore)):
+        before = host_values(t)
+        call(plan, 3, 0.0)
+        torch.cuda.synchronize()
+        got, want = host_values(t), oracle_call(before, g, 3, 0.0, dtype)
+        bits = got.view(np.uint16 if dtype == "bf16" else np.uint32)
+        wbits = want.view(np.uint16 if dtype == "bf16" else np.uint32)
+        if dtype == "bf16":
+            nan = np.isnan((want.astype(np.uint32) << 16).view(np.float32))
+        else:
+            nan = np.isnan(want)
+        assert np.array_equal(bits[~nan], wbits[~nan])
+        assert np.array_equal(bits[~nan & (vals != 0)], host_bits(before, dtype)[~nan & (vals != 0)])
+        assert np.all(np.isnan((bits.astype(np.uint32) << 16).view(np.float32) if dtype == "bf16"
+                               else got)[nan])
+    plan.close()
+
+
+def host_bits(v, dtype):
+    return v.view(np.uint16 if dtype == "bf16" else np.uint32)
+
+
+@pytest.mark.parametrize("dtype", ["bf16", "f32"])
+def test_zero_coefficients_are_skipped_and_repeated_seeds_add(es, oracle, dtype):
+    a = make_params(dtype, RAGGED[:6], seed=13)
+    b = [x.clone() for x in a]
+    plan_a, segs = build_plan(es, a)
+    plan_b, _ = build_plan(es, b, [s.index_base for s in segs])
+    es.es_update(plan_a, [11, 12, 13, 14], np.array([2e-4, 0.0, -1e-4, 0.0], np.float32))
+    es.es_update(plan_b, [11, 13], np.array([2e-4, -1e-4], np.float32))
+    torch.cuda.synchronize()
+    for x, y in zip(a, b):
+        assert torch.equal(_int_view(x), _int_view(y))
+    # the same seed twice contributes twice
+    before = [host_values(x) for x in a]
+    seeds = np.array([21, 21, 22], dtype=np.uint64)
+    coeffs = np.array([1e-4, 3e-4, -2e-4], np.float32)
+    es.es_update(plan_a, seeds, coeffs)
+    torch.cuda.synchronize()
+    for x, s, h in zip(a, segs, before):
+        g = indices([s])[0]
+        tol = noise_abs_tol([oracle.noise_at(int(k), g) for k in seeds], coeffs)
+        compare(dtype, host_values(x), oracle.update(h, g, seeds, coeffs, dtype), "repeated seed", tol)
+    plan_a.close()
+    plan_b.close()
