@@ -245,3 +245,65 @@ def test_all_equal_rewards_leave_the_4b_set_bit_identical(es):
     plan.close()
     del params, ref, plan
     _release()
+
+
+def test_bench_step_on_the_27b_set_equals_the_oracle_checked_separate_calls(es, oracle):
+    # The benchmarked generation exactly as bench.py times it: its flat
+    # single-allocation layout, its plan and its fused loop (bench.start_loop,
+    # then bench.run_step: es_restore_perturb x 29, es_restore,
+    # es_update_perturb). A twin copy of the set runs the same generation as
+    # separate calls, each checked against the oracle on sampled elements from
+    # the state before it; at the end all 22.7e9 parameters of the two copies
+    # must be bit-identical.
+    import bench
+    wl = I.WORKLOADS["qwen27b"]
+    specs = I.shapes_for("qwen27b")
+    n = wl.population
+    flat, params = I.init_params_flat(specs, torch.bfloat16, "cuda", seed=0)
+    twin_flat = flat.clone()
+    offs = I.flat_offsets(specs)
+    twin = [twin_flat[o:o + s.numel] for s, o in zip(specs, offs)]
+    plan = es.plan_from_tensors(params)
+    segs = es.segments_from_tensors(twin)
+    twin_plan = es.plan_from_tensors(twin, [s.index_base for s in segs])
+    smp = Sampled(twin, segs, 30, seed=41)
+    stream = torch.cuda.current_stream().cuda_stream
+
+    def sigma_at(t):
+        return float(np.float32(es.es_sigma_cosine(wl.sigma, bench.SIGMA_FINAL["qwen27b"], t,
+                                                  bench.SCHEDULE_T)))
+
+    sigma, sigma_next = sigma_at(0), sigma_at(1)
+    bench.start_loop(es, plan, wl, 0, n, sigma, stream, True)
+    launches = bench.run_step(es, plan, wl, 0, n, sigma, sigma_next, stream, None, True)
+    assert launches == n + 1
+
+    seeds, rewards = bench.generation_inputs(wl, 0, n)
+    coeffs = es.es_update_coeffs(es.es_normalize_rewards(rewards, 1e-8), wl.alpha, sigma,
+                                 es.ES_SCALE_PAPER)
+    next_seed = int(bench.generation_inputs(wl, 1, n)[0][0])
+
+    def checked(call, oracle_call, seed_list, coeff_list, what):
+        before = smp.gather()
+        call()
+        torch.cuda.synchronize()
+        want = oracle_call(before)
+        tol = noise_abs_tol([oracle.noise_at(int(s), smp.g) for s in seed_list], coeff_list)
+        assert_bf16_within_ulp(smp.gather(), want, what, abs_tol=tol)
+
+    for i, s in enumerate(seeds):
+        s = int(s)
+        checked(lambda: es.es_perturb(twin_plan, s, sigma),
+                lambda b: oracle.perturb(b, smp.g, s, sigma, "bf16"), [s], [sigma], f"perturb {i}")
+        checked(lambda: es.es_restore(twin_plan, s, sigma),
+                lambda b: oracle.restore(b, smp.g, s, sigma, "bf16"), [s], [sigma], f"restore {i}")
+    checked(lambda: es.es_update(twin_plan, seeds, coeffs),
+            lambda b: oracle.update(b, smp.g, seeds, coeffs, "bf16"), seeds, coeffs, "update")
+    checked(lambda: es.es_perturb(twin_plan, next_seed, sigma_next),
+            lambda b: oracle.perturb(b, smp.g, next_seed, sigma_next, "bf16"), [next_seed],
+            [sigma_next], "next perturb")
+    assert torch.equal(flat.view(torch.int16), twin_flat.view(torch.int16))
+    plan.close()
+    twin_plan.close()
+    del flat, twin_flat, params, twin, smp, plan, twin_plan
+    _release()
