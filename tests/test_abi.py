@@ -189,3 +189,41 @@ def test_normalize_rewards_in_place(E, oracle):
 def test_assign_index_bases_overflow_returns_zero(E):
     segs = [E.Segment(0, 2**63), E.Segment(0, 2**63 + 16)]
     assert E.es_assign_index_bases(segs) == 0
+
+
+def test_last_error_is_per_thread(E):
+    # Each thread provokes a different validation error (no device call is
+    # reached) and must read back its own detail, whatever the other threads
+    # do meanwhile: es_last_error() is thread-local.
+    import threading
+    S = E.Segment
+    cases = {
+        "align": ([S(0x1001, 16, 0)], "16-byte aligned"),
+        "base": ([S(0x1000, 16, 3)], "multiple of 8"),
+        "overlap": ([S(0x1000, 16, 0), S(0x2000, 16, 8)], "overlap in index space"),
+        "empty": ([S(0x1000, 0, 0)], "zero numel"),
+    }
+    errors = []
+    barrier = threading.Barrier(len(cases))
+
+    def worker(name, segs, expect):
+        try:
+            barrier.wait()
+            for _ in range(200):
+                try:
+                    E.es_plan_create(segs, E.ES_BF16)
+                except E.EsError:
+                    pass
+                msg = E.es_last_error()
+                if expect not in msg:
+                    errors.append((name, msg))
+                    return
+        except Exception as exc:  # pragma: no cover
+            errors.append((name, repr(exc)))
+
+    threads = [threading.Thread(target=worker, args=(k, s, e)) for k, (s, e) in cases.items()]
+    for t in threads:
+        t.start()
+    for t in threads:
+        t.join()
+    assert not errors, errors

@@ -551,3 +551,37 @@ def test_zero_coefficients_are_skipped_and_repeated_seeds_add(es, oracle, dtype)
         compare(dtype, host_values(x), oracle.update(h, g, seeds, coeffs, dtype), "repeated seed", tol)
     plan_a.close()
     plan_b.close()
+
+
+def test_two_plans_on_two_streams_equal_the_sequential_result(es):
+    # Launches on two streams with no synchronisation between them (distinct
+    # plans over distinct tensors) give bit-identically what the same calls
+    # give one after the other on one stream.
+    a = make_params("bf16", RAGGED, seed=20)
+    b = make_params("bf16", RAGGED[::-1], seed=21)
+    a_ref = [t.clone() for t in a]
+    b_ref = [t.clone() for t in b]
+    plans = [build_plan(es, ts)[0] for ts in (a, b, a_ref, b_ref)]
+    seeds = np.arange(40, 48, dtype=np.uint64)
+    coeffs = np.linspace(-2e-4, 3e-4, 8).astype(np.float32)
+
+    def generation(plan, stream):
+        for s in seeds:
+            es.es_perturb(plan, int(s), 1e-3, stream)
+            es.es_restore(plan, int(s), 1e-3, stream)
+        es.es_update(plan, seeds, coeffs, stream)
+
+    s1, s2 = torch.cuda.Stream(), torch.cuda.Stream()
+    torch.cuda.synchronize()
+    for _ in range(3):
+        generation(plans[0], s1.cuda_stream)
+        generation(plans[1], s2.cuda_stream)
+    torch.cuda.synchronize()
+    for _ in range(3):
+        generation(plans[2], None)
+        generation(plans[3], None)
+    torch.cuda.synchronize()
+    for x, y in zip(a + b, a_ref + b_ref):
+        assert torch.equal(_int_view(x), _int_view(y))
+    for p in plans:
+        p.close()
