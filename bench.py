@@ -37,7 +37,6 @@ UNIT = "param*seed/s"
 SIGMA_FINAL = {"qwen27b": 2.5e-4, "qwen4b": 5e-4, "qwen4b_f32": 5e-4, "qwen4b_4layer": 5e-4,
                "toy": 1e-3}
 SCHEDULE_T = 100
-CPU_SAMPLE = 1 << 21
 
 
 def parse():
@@ -168,6 +167,9 @@ class ClockSampler:
 
 # --- the step -------------------------------------------------------------------------------
 
+L2_BYTES = 129 * 1024 * 1024     # GB300 L2
+
+
 def workload_config(workload: str, n: int, world: int) -> dict:
     """The `config` object of the JSON line (shared by both arms)."""
     wl = I.WORKLOADS[workload]
@@ -176,7 +178,10 @@ def workload_config(workload: str, n: int, world: int) -> dict:
     esize = 2 if wl.dtype == "bf16" else 4
     return {"workload": workload, "params": P, "population": n, "storage": wl.dtype,
             "segments": len(specs), "description": wl.description, "alpha": wl.alpha,
-            "l2": "inputs larger than L2 (%.1f GB of parameters)" % (P * esize / 1e9),
+            "l2": ("inputs larger than L2 (%.1f GB of parameters)" % (P * esize / 1e9)
+                   if P * esize > L2_BYTES else
+                   "inputs smaller than L2 (%.1f MB of parameters): not an HBM measurement"
+                   % (P * esize / 1e6)),
             "parallelism": "replicas" if world > 1 else "single GPU"}
 
 
@@ -754,14 +759,14 @@ def run_e2e(args, torch, es, plan, flat, params, wl, n, esize, sigma_at, s_handl
 
 # --- CPU oracle (cpu_baseline leg and the reference arm) ---------------------------------
 
-def oracle_sample_step(workload: str, n: int, sigma: float, sample: int, step: int):
-    """One ES generation of the oracle on the first `sample` parameters of the
-    workload's first weight tensor. Returns elapsed seconds."""
+def oracle_generation(workload: str, n: int, sigma: float, lo: int, count: int, step: int):
+    """One ES generation (N perturb + restore pairs, the update) of the oracle on
+    parameters [lo, lo + count) of the workload's first weight tensor. Returns
+    (seconds of oracle work, parameters)."""
     from oracle import oracle as O
     wl = I.WORKLOADS[workload]
-    specs = I.shapes_for(workload)
-    g = np.arange(min(sample, specs[0].numel), dtype=np.uint64)
-    theta32 = I.normal_f32(g.size, 0, 0.02)
+    g = np.arange(lo, lo + count, dtype=np.uint64)
+    theta32 = I.normal_f32(g.size, lo, 0.02)
     dt = "bf16" if wl.dtype == "bf16" else "f32"
     if dt == "bf16":
         import torch
@@ -778,12 +783,79 @@ def oracle_sample_step(workload: str, n: int, sigma: float, sample: int, step: i
     return time.perf_counter() - t0, g.size
 
 
-def cpu_baseline(workload, n, sigma, sample=CPU_SAMPLE):
-    secs, m = oracle_sample_step(workload, n, sigma, sample, 0)
-    return {"value": m * n / secs, "unit": UNIT, "cores": 1, "kind": "oracle",
-            "sample": f"one generation (N={n} perturb+restore, update) on the first {m} "
-                      f"parameters of the {workload} set, single-threaded plain-C oracle; "
-                      f"{secs:.1f} s"}
+def _oracle_worker_init():
+    import torch  # noqa: F401  (bf16 conversion of the inputs, loaded before timing)
+    from oracle import oracle as O
+    O.lib()
+
+
+def _oracle_task(a):
+    return oracle_generation(*a)
+
+
+def host_cores() -> int:
+    try:
+        return len(os.sched_getaffinity(0))
+    except AttributeError:  # pragma: no cover
+        return os.cpu_count() or 1
+
+
+def cpu_model() -> str:
+    try:
+        out = subprocess.run(["lscpu"], capture_output=True, text=True, timeout=10).stdout
+        for line in out.splitlines():
+            if line.startswith("Model name:"):
+                return line.split(":", 1)[1].strip()
+    except (OSError, subprocess.SubprocessError):
+        pass
+    return "unknown"
+
+
+class OraclePool:
+    """The unchanged oracle on every host core: one spawned worker per core,
+    each running whole generations on its own slice of the parameters (the
+    step is elementwise, so slices are independent). Spawned, never forked, so
+    it is safe after CUDA has been initialised."""
+
+    def __init__(self, workers: int):
+        import multiprocessing as mp
+        self.workers = workers
+        self.pool = mp.get_context("spawn").Pool(workers, initializer=_oracle_worker_init)
+
+    def generation(self, workload, n, sigma, per_worker, step):
+        """Wall seconds of one generation over workers x per_worker parameters
+        (fewer where the tensor is smaller), and the parameters covered."""
+        numel = I.shapes_for(workload)[0].numel
+        tasks = [(workload, n, sigma, lo, min(per_worker, numel - lo), step)
+                 for lo in range(0, min(numel, self.workers * per_worker), per_worker)]
+        t0 = time.perf_counter()
+        res = self.pool.map(_oracle_task, tasks, chunksize=1)
+        return time.perf_counter() - t0, sum(m for _, m in res)
+
+    def close(self):
+        self.pool.close()
+        self.pool.join()
+
+
+def cpu_baseline(workload, n, sigma):
+    """The oracle on all host cores over about 2^22 parameters (10-30 s of CPU
+    work), plus its single-thread rate on 2^20 parameters."""
+    cores = host_cores()
+    per_worker = max(1 << 16, (1 << 22) // cores)
+    pool = OraclePool(cores)
+    try:
+        pool.generation(workload, n, sigma, 1 << 12, 0)            # workers up and warm
+        wall, m = pool.generation(workload, n, sigma, per_worker, 0)
+    finally:
+        pool.close()
+    secs1, m1 = oracle_generation(workload, n, sigma, 0, 1 << 20, 0)
+    return {"value": m * n / wall, "unit": UNIT, "cores": cores, "kind": "oracle",
+            "sample": f"one generation (N={n} perturb+restore, update) on {m} parameters of "
+                      f"the {workload} set's first weight tensor, split over {cores} spawned "
+                      f"workers of the unchanged plain-C oracle; {wall:.1f} s wall",
+            "single_thread": {"value": m1 * n / secs1, "cores": 1, "params": m1,
+                              "seconds": secs1},
+            "cpu_model": cpu_model()}
 
 
 def run_reference(args, rank, world):
@@ -792,23 +864,29 @@ def run_reference(args, rank, world):
     wl = I.WORKLOADS[args.workload]
     n = args.population or wl.population
     sigma = float(np.float32(wl.sigma))
-    sample = 1 << 17
-    for w in range(args.warmup):
-        oracle_sample_step(args.workload, n, sigma, sample, w)
-    tot, m = 0.0, 0
-    for k in range(args.steps):
-        secs, m = oracle_sample_step(args.workload, n, sigma, sample, args.warmup + k)
-        tot += secs
-    value = m * n * args.steps / tot
-    desc = (f"each step: one generation (N={n}) of the plain-C oracle on the first {m} "
-            f"parameters of the {args.workload} set, single-threaded")
+    cores = host_cores()
+    per_worker = 1 << 17
+    pool = OraclePool(cores)
+    try:
+        for w in range(args.warmup):
+            pool.generation(args.workload, n, sigma, per_worker, w)
+        tot, m = 0.0, 0
+        for k in range(args.steps):
+            secs, m = pool.generation(args.workload, n, sigma, per_worker, args.warmup + k)
+            tot += secs
+    finally:
+        pool.close()
+    value = m * n * args.steps / tot if tot > 0 else 0.0
+    desc = (f"each step: one generation (N={n}) of the unchanged plain-C oracle on {m} "
+            f"parameters of the {args.workload} set, split over {cores} spawned workers")
     out = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world,
-           "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * tot / args.steps,
+           "steps": args.steps, "warmup": args.warmup,
+           "ms_per_step": 1e3 * tot / args.steps if args.steps else 0.0,
            "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
            "dtype": "f64", "data": "synthetic", "impl": "reference",
            "config": dict(workload_config(args.workload, n, 1), sigma=sigma, sample_params=m),
-           "cpu_baseline": {"value": value, "unit": UNIT, "cores": 1, "kind": "oracle",
-                            "sample": desc},
+           "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores, "kind": "oracle",
+                            "sample": desc, "cpu_model": cpu_model()},
            "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0,
                    "d2h_bytes_per_step": 0},
            "gpu_launches": 0}
