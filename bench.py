@@ -57,8 +57,15 @@ def parse():
                         "(default workload qwen4b) and print one JSON line with every point")
     p.add_argument("--populations", default="1,2,4,8,16,32,64,128",
                    help="comma-separated N values of --sweep")
+    p.add_argument("--replay", action="store_true",
+                   help="instead of the step: K logged generations applied by one es_replay "
+                        "against K es_update calls (default workload qwen4b)")
+    p.add_argument("--generations", type=int, default=16, help="K of --replay")
+    p.add_argument("--antithetic", action="store_true",
+                   help="instead of the step: a generation of N/2 antithetic pairs (the +/- "
+                        "flip as one es_restore_perturb on one seed)")
     args = p.parse_args()
-    if args.sweep and "--workload" not in " ".join(sys.argv):
+    if (args.sweep or args.replay) and "--workload" not in " ".join(sys.argv):
         args.workload = "qwen4b"
     return args
 
@@ -579,6 +586,178 @@ def run_sweep(args, rank, world, dist):
         print(json.dumps(out), flush=True)
 
 
+def _timed(torch, stream, fn, reps):
+    """Mean milliseconds of fn() over reps runs, CUDA events on `stream`."""
+    e0 = torch.cuda.Event(enable_timing=True)
+    e1 = torch.cuda.Event(enable_timing=True)
+    torch.cuda.synchronize()
+    e0.record(stream)
+    for _ in range(reps):
+        fn()
+    e1.record(stream)
+    torch.cuda.synchronize()
+    return e0.elapsed_time(e1) / reps
+
+
+def _rates(P, gaussians_per_param, bytes_total, ms, peaks_):
+    imul_peak, gauss_peak, shared_peak, _, _, hbm_gbs, _ = peaks_
+    gps = gaussians_per_param * P / (ms / 1e3)
+    gbs = bytes_total / (ms / 1e3) / 1e9
+    return {"ms": ms, "gauss_per_s": gps, "gbs": gbs, "hbm_frac": gbs / hbm_gbs,
+            "alu_frac": gps / gauss_peak, "imul_mufu_frac": gps / shared_peak}
+
+
+def run_replay(args, rank, world, dist):
+    """es_replay of K logged generations (N seeds each) in one pass over the
+    parameters, against the same K generations as K es_update calls."""
+    import torch
+    from paper_2608_17310_gb300 import build, esopt as es
+
+    build.build_library()
+    dev_index = torch.cuda.current_device()
+    torch.cuda.init()
+    wl = I.WORKLOADS[args.workload]
+    n = args.population or wl.population
+    K = args.generations
+    specs = I.shapes_for(args.workload)
+    dtype = torch.bfloat16 if wl.dtype == "bf16" else torch.float32
+    esize = 2 if wl.dtype == "bf16" else 4
+    flat, params = I.init_params_flat(specs, dtype, "cuda", seed=0)
+    plan = es.plan_from_tensors(params)
+    P = plan.numel
+    stream = torch.cuda.current_stream()
+    sh = stream.cuda_stream
+    sigma = float(np.float32(wl.sigma))
+    seeds, coeffs = [], []
+    for g in range(K):
+        # N(0, 1) rewards used as the normalised rewards (as in the sweep): no
+        # generation of the log degenerates to an all-zero update
+        seeds.append(I.population_seeds(n, generation=g))
+        coeffs.append(es.es_update_coeffs(I.rewards("normal", n, seed=g), wl.alpha, sigma,
+                                          es.ES_SCALE_PAPER))
+    all_seeds, all_coeffs = np.concatenate(seeds), np.concatenate(coeffs)
+    counts = np.full(K, n, dtype=np.int32)
+    # launches es_replay makes: a pass holds <= ES_MAX_SEEDS non-zero seeds and
+    # <= 256 generations, and breaks only between generations
+    passes, in_pass, gens = 0, 0, 0
+    for g in range(K):
+        nz = int(np.count_nonzero(coeffs[g]))
+        if nz and (in_pass + nz > es.ES_MAX_SEEDS or gens == 256):
+            passes, in_pass, gens = passes + 1, 0, 0
+        if nz:
+            in_pass, gens = in_pass + nz, gens + 1
+    passes += 1 if gens else 0
+
+    def replay():
+        es.es_replay(plan, all_seeds, all_coeffs, counts, sh)
+
+    def separate():
+        for g in range(K):
+            es.es_update(plan, seeds[g], coeffs[g], sh)
+
+    pk = alu_peaks(torch, dev_index)
+    with ClockSampler(dev_index) as clk:
+        for _ in range(args.warmup):
+            replay()
+            separate()
+        ms_r = _timed(torch, stream, replay, args.steps)
+        ms_s = _timed(torch, stream, separate, args.steps)
+    plan.close()
+    live = int(sum(np.count_nonzero(c) for c in coeffs))      # seeds that are applied
+    live_gens = int(sum(1 for c in coeffs if np.any(c != 0)))  # es_update calls that launch
+    r = _rates(P, live, passes * 2 * esize * P, ms_r, pk)
+    sep = _rates(P, live, live_gens * 2 * esize * P, ms_s, pk)
+    out = {"mode": "replay", "metric": "seed-log replay param*seed/s", "unit": UNIT,
+           "value": P * live / (ms_r / 1e3), "n_gpus": 1, "steps": args.steps,
+           "warmup": args.warmup, "ms_per_step": ms_r, "higher_is_better": True,
+           "dtype": "f32", "data": "synthetic",
+           "config": dict(workload_config(args.workload, n, 1), generations=K,
+                          seeds_per_replay=live, replay_passes=passes,
+                          rewards="N(0,1) used as the normalised rewards"),
+           "replay": r, "separate_updates": sep, "speedup": ms_s / ms_r,
+           "gpu_launches": args.steps * (passes + live_gens), "clocks": clk.summary()}
+    if rank == 0:
+        print(json.dumps(out), flush=True)
+
+
+def run_antithetic(args, rank, world, dist):
+    """A generation of N/2 antithetic pairs, steady state: each pair's flip from
+    +sigma eps_i to -sigma eps_i is one es_restore_perturb on one seed (noise
+    generated once); between pairs es_restore_perturb moves to the next seed;
+    the generation ends with es_restore and es_update_perturb over the folded
+    per-pair coefficients."""
+    import torch
+    from paper_2608_17310_gb300 import build, esopt as es
+
+    build.build_library()
+    dev_index = torch.cuda.current_device()
+    torch.cuda.init()
+    wl = I.WORKLOADS[args.workload]
+    pairs = (args.population or wl.population) // 2
+    specs = I.shapes_for(args.workload)
+    dtype = torch.bfloat16 if wl.dtype == "bf16" else torch.float32
+    esize = 2 if wl.dtype == "bf16" else 4
+    flat, params = I.init_params_flat(specs, dtype, "cuda", seed=0)
+    plan = es.plan_from_tensors(params)
+    P = plan.numel
+    stream = torch.cuda.current_stream()
+    sh = stream.cuda_stream
+    sigma0, sigmaT = wl.sigma, SIGMA_FINAL.get(args.workload, wl.sigma)
+
+    def sigma_at(t):
+        return float(np.float32(es.es_sigma_cosine(sigma0, sigmaT, t, SCHEDULE_T)))
+
+    def inputs(t):
+        seeds = I.population_seeds(pairs, generation=t)
+        rewards = I.rewards("uniform", 2 * pairs, seed=t)
+        return seeds, rewards
+
+    launches = [0]
+
+    def step(t):
+        sigma, sigma_next = sigma_at(t), sigma_at(t + 1)
+        seeds, rewards = inputs(t)
+        for i, sd in enumerate(seeds):
+            es.es_restore_perturb(plan, int(sd), sigma, int(sd), -sigma, sh)      # + -> -
+            if i + 1 < pairs:
+                es.es_restore_perturb(plan, int(sd), -sigma, int(seeds[i + 1]), sigma, sh)
+            else:
+                es.es_restore(plan, int(sd), -sigma, sh)
+        rhat = es.es_normalize_rewards(rewards, 1e-8)
+        coeffs = es.es_fold_antithetic(rhat[:pairs], rhat[pairs:], wl.alpha, sigma,
+                                       es.ES_SCALE_PAPER)
+        es.es_update_perturb(plan, seeds, coeffs, int(inputs(t + 1)[0][0]), sigma_next, sh)
+        launches[0] += 2 * pairs + 1
+
+    es.es_perturb(plan, int(inputs(0)[0][0]), sigma_at(0), sh)
+    pk = alu_peaks(torch, dev_index)
+    for w in range(args.warmup):
+        step(w)
+    launches[0] = 0
+    t_box = [args.warmup]
+
+    def timed_step():
+        step(t_box[0])
+        t_box[0] += 1
+
+    with ClockSampler(dev_index) as clk:
+        ms = _timed(torch, stream, timed_step, args.steps)
+    plan.close()
+    members = 2 * pairs
+    gauss = pairs * 1 + (pairs - 1) * 2 + 1 + (pairs + 1)
+    passes = 2 * pairs + 1
+    out = {"mode": "antithetic", "metric": "ES step param*member/s, antithetic pairs",
+           "unit": "param*member/s", "value": P * members / (ms / 1e3), "n_gpus": 1,
+           "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms,
+           "higher_is_better": True, "dtype": "f32", "data": "synthetic",
+           "config": dict(workload_config(args.workload, members, 1), pairs=pairs,
+                          gaussians_per_param=gauss, passes=passes),
+           "rates": _rates(P, gauss, passes * 2 * esize * P, ms, pk),
+           "gpu_launches": launches[0], "clocks": clk.summary()}
+    if rank == 0:
+        print(json.dumps(out), flush=True)
+
+
 class PinnedHostBuffer:
     """Page-locked host memory for the e2e copies: anonymous mmap with
     transparent huge pages requested (madvise), registered with
@@ -904,6 +1083,10 @@ def main():
     try:
         if args.sweep:
             run_sweep(args, rank, world, dist)
+        elif args.replay:
+            run_replay(args, rank, world, dist)
+        elif args.antithetic:
+            run_antithetic(args, rank, world, dist)
         else:
             run_ours(args, rank, world, dist)
     finally:
