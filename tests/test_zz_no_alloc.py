@@ -63,3 +63,25 @@ def test_noalloc_rejects_more_segments_than_its_static_table(es):
         es.es_perturb_noalloc(segs, es.ES_BF16, 1, 1e-3)
     assert ei.value.status == es.ES_ERR_INVALID_ARG
     assert "ES_STATIC_MAX_SEGMENTS" in str(ei.value)
+
+
+def test_noalloc_at_its_segment_limit_matches_the_plan(es):
+    # Exactly ES_STATIC_MAX_SEGMENTS ragged segments (1 .. 600 elements, 16-byte
+    # aligned views of one buffer): the whole static table is in use.
+    n = es.ES_STATIC_MAX_SEGMENTS
+    rng = np.random.default_rng(31)
+    sizes = rng.integers(1, 601, size=n)
+    offs = np.concatenate([[0], np.cumsum((sizes + 7) // 8 * 8)])
+    flat = torch.from_numpy((0.02 * rng.standard_normal(int(offs[-1]))).astype(np.float32))
+    flat = flat.to(torch.bfloat16).cuda()
+    twin = flat.clone()
+    a = [flat[int(o):int(o) + int(m)] for o, m in zip(offs[:-1], sizes)]
+    b = [twin[int(o):int(o) + int(m)] for o, m in zip(offs[:-1], sizes)]
+    plan = es.plan_from_tensors(a)
+    segs_b = es.segments_from_tensors(b, [s.index_base for s in es.segments_from_tensors(a)])
+    for seed, sigma in ((2**40 + 3, 1e-3), (2**40 + 3, -1e-3), (77, 5e-4)):
+        es.es_perturb(plan, seed, sigma)
+        es.es_perturb_noalloc(segs_b, es.ES_BF16, seed, sigma)
+        torch.cuda.synchronize()
+        assert torch.equal(flat.view(torch.int16), twin.view(torch.int16))
+    plan.close()
