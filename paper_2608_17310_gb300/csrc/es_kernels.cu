@@ -117,21 +117,49 @@ __device__ __forceinline__ auto make_gen(PhiloxKey key, uint32_t j_hi) {
   else return AnyGen{key};
 }
 
+// How each Philox block becomes theta updates. The forms give bit-identical
+// values: a packed two-wide FP32 instruction rounds each half exactly like the
+// scalar one. They differ only in instruction mix, which moves work between the
+// FMA pipe's halves. Each kernel uses the form measured fastest for it:
+//   kScalar     scalar transform (polar) and scalar FMAs;
+//   kPackedFma  scalar transform, packed FMAs into theta or the accumulator;
+//   kPacked     packed transform (polar2) and packed FMAs.
+enum class NoiseForm { kScalar, kPackedFma, kPacked };
+
 // f[k] += scale * eps[g0 + k] for the V elements from global index g0
 // (g0 % 4 == 0), with scale folded into each pair's radius.
-template <int V, class Gen>
+template <NoiseForm kForm, int V, class Gen>
 __device__ __forceinline__ void add_scaled_noise(const Gen& gen, uint64_t g0, float scale,
                                                  float (&f)[V]) {
 #pragma unroll
   for (int b = 0; b < V / 4; ++b) {
     const uint4 x = gen.block((g0 >> 2) + b);
-    const Polar p = polar(x.x, x.y);
-    const Polar q = polar(x.z, x.w);
-    const float sp = -(scale * p.r), sq = -(scale * q.r);
-    f[4 * b + 0] = fmaf(sp, p.c, f[4 * b + 0]);
-    f[4 * b + 1] = fmaf(sp, p.s, f[4 * b + 1]);
-    f[4 * b + 2] = fmaf(sq, q.c, f[4 * b + 2]);
-    f[4 * b + 3] = fmaf(sq, q.s, f[4 * b + 3]);
+    if constexpr (kForm == NoiseForm::kScalar) {
+      const Polar p = polar(x.x, x.y);
+      const Polar q = polar(x.z, x.w);
+      const float sp = -(scale * p.r), sq = -(scale * q.r);
+      f[4 * b + 0] = fmaf(sp, p.c, f[4 * b + 0]);
+      f[4 * b + 1] = fmaf(sp, p.s, f[4 * b + 1]);
+      f[4 * b + 2] = fmaf(sq, q.c, f[4 * b + 2]);
+      f[4 * b + 3] = fmaf(sq, q.s, f[4 * b + 3]);
+    } else {
+      Polar2 p;
+      if constexpr (kForm == NoiseForm::kPacked) {
+        p = polar2(x);
+      } else {
+        const Polar a = polar(x.x, x.y), c = polar(x.z, x.w);
+        p = Polar2{make_float2(a.r, c.r), make_float2(a.c, c.c), make_float2(a.s, c.s)};
+      }
+      const float2 sr = __fmul2_rn(make_float2(-scale, -scale), p.r);   // -(scale * r)
+      const float2 lo = __ffma2_rn(make_float2(sr.x, sr.x), make_float2(p.c.x, p.s.x),
+                                   make_float2(f[4 * b + 0], f[4 * b + 1]));
+      const float2 hi = __ffma2_rn(make_float2(sr.y, sr.y), make_float2(p.c.y, p.s.y),
+                                   make_float2(f[4 * b + 2], f[4 * b + 3]));
+      f[4 * b + 0] = lo.x;
+      f[4 * b + 1] = lo.y;
+      f[4 * b + 2] = hi.x;
+      f[4 * b + 3] = hi.y;
+    }
   }
 }
 
@@ -198,6 +226,8 @@ template <class Io, bool kTwo, bool kSame, bool kUniformHi>
 __device__ __forceinline__ void axpy_tile(const TileRef<Io>& r, PhiloxKey key, float scale,
                                           PhiloxKey key2, float scale2) {
   constexpr int V = Io::kVec, U = Io::kVecs;
+  // the two-seed pass is fastest fully packed, the one-seed pass scalar
+  constexpr NoiseForm kAxpyForm = kTwo ? NoiseForm::kPacked : NoiseForm::kScalar;
   typename Io::Scalar* const base = r.base;
   const uint64_t numel = r.numel, index_base = r.index_base, t0 = r.t0;
   const uint32_t j_hi = static_cast<uint32_t>((index_base + t0) >> 34);
@@ -225,10 +255,10 @@ __device__ __forceinline__ void axpy_tile(const TileRef<Io>& r, PhiloxKey key, f
     if (kSame) {
       add_scaled_noise_twice<Io, V>(gen, index_base + e, scale, scale2, f);
     } else {
-      add_scaled_noise<V>(gen, index_base + e, scale, f);
+      add_scaled_noise<kAxpyForm, V>(gen, index_base + e, scale, f);
       if (kTwo) {
         Io::round_trip(f);
-        add_scaled_noise<V>(gen2, index_base + e, scale2, f);
+        add_scaled_noise<kAxpyForm, V>(gen2, index_base + e, scale2, f);
       }
     }
     if (full) {
@@ -296,7 +326,7 @@ __device__ __forceinline__ void update_tile_single(typename Io::Scalar* base, ui
       for (int q = 0; q < G; ++q) {
         const uint64_t e = t0 + static_cast<uint64_t>((u0 + q) * kBlockThreads + threadIdx.x) * V;
         if (e >= numel) continue;
-        add_scaled_noise<V>(gen, index_base + e, c, acc[q]);
+        add_scaled_noise<NoiseForm::kPackedFma, V>(gen, index_base + e, c, acc[q]);
       }
     }
 #pragma unroll
@@ -316,7 +346,7 @@ __device__ __forceinline__ void update_tile_single(typename Io::Scalar* base, ui
       for (int k = 0; k < V; ++k) f[k] = f[k] + acc[q][k];
       if (kPerturb) {
         Io::round_trip(f);
-        add_scaled_noise<V>(pgen, index_base + e, args.pscale, f);
+        add_scaled_noise<NoiseForm::kPackedFma, V>(pgen, index_base + e, args.pscale, f);
       }
       if (full) {
         *reinterpret_cast<uint4*>(base + e) = Io::pack(f);
@@ -369,7 +399,7 @@ __device__ __forceinline__ void update_tile(typename Io::Scalar* base, uint64_t 
         for (int q = 0; q < G; ++q) {
           const uint64_t e = t0 + static_cast<uint64_t>((u0 + q) * kBlockThreads + threadIdx.x) * V;
           if (e >= numel) continue;
-          add_scaled_noise<V>(gen, index_base + e, c, acc[q]);
+          add_scaled_noise<NoiseForm::kPackedFma, V>(gen, index_base + e, c, acc[q]);
         }
       }
 #pragma unroll
@@ -389,7 +419,7 @@ __device__ __forceinline__ void update_tile(typename Io::Scalar* base, uint64_t 
         if (e >= numel) continue;
         float f[V];
         Io::unpack(v[q], f);
-        add_scaled_noise<V>(gen, index_base + e, args.pscale, f);
+        add_scaled_noise<NoiseForm::kPackedFma, V>(gen, index_base + e, args.pscale, f);
         v[q] = Io::pack(f);
       }
     }

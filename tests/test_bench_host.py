@@ -48,5 +48,5 @@ def test_pipe_occupancy_file_is_keyed_by_the_current_code():
             if line.strip() and not line.startswith("#")]
     assert {r[0] for r in rows} == {"restore_perturb", "update_perturb", "update"}
     if all(r[3] == bench.kernel_code_digest() for r in rows):
-        assert occ is not None and 90.0 < occ["sum_pct"] < 105.0
+        assert occ is not None and 90.0 < occ["sum_pct"] < 115.0
     assert bench.pipe_occupancy("restore") is None
