@@ -637,15 +637,19 @@ def run_replay(args, rank, world, dist):
                                           es.ES_SCALE_PAPER))
     all_seeds, all_coeffs = np.concatenate(seeds), np.concatenate(coeffs)
     counts = np.full(K, n, dtype=np.int32)
-    # launches es_replay makes: a pass holds <= ES_MAX_SEEDS non-zero seeds and
-    # <= 256 generations, and breaks only between generations
+    # launches es_replay makes: generations of fewer than 4 non-zero seeds
+    # share a pass (<= ES_MAX_SEEDS seeds, <= 256 generations); a larger one
+    # has a pass of its own; passes break only between generations
     passes, in_pass, gens = 0, 0, 0
     for g in range(K):
         nz = int(np.count_nonzero(coeffs[g]))
-        if nz and (in_pass + nz > es.ES_MAX_SEEDS or gens == 256):
+        own = nz >= 4
+        if nz and gens and (own or in_pass + nz > es.ES_MAX_SEEDS or gens == 256):
             passes, in_pass, gens = passes + 1, 0, 0
         if nz:
             in_pass, gens = in_pass + nz, gens + 1
+        if own:
+            passes, in_pass, gens = passes + 1, 0, 0
     passes += 1 if gens else 0
 
     def replay():

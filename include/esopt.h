@@ -253,9 +253,10 @@ es_status_t es_update_perturb(es_plan_t plan, const uint64_t* seeds, const float
  *   theta[g] <- round(theta[g] + sum_{i in generation g} coeffs[i] * eps_{seeds[i]}[g]),
  * bit-identical to one es_update per generation. `seeds` and `coeffs` hold
  * the generations back to back; counts[g] (1 .. ES_MAX_SEEDS) is the size of
- * generation g. Up to 256 generations and ES_MAX_SEEDS seeds are fused per
- * pass over theta; longer logs take several passes, split between
- * generations. Host arrays; asynchronous on `stream`. All arguments are
+ * generation g. Generations of fewer than 4 non-zero seeds are fused, up to
+ * 256 generations and ES_MAX_SEEDS seeds per pass over theta; a larger
+ * generation gets a pass of its own, which computes it faster. Passes split
+ * only between generations. Host arrays; asynchronous on `stream`. All arguments are
  * checked before the first pass; if a launch then fails (ES_ERR_CUDA), the
  * passes before it have been applied.
  * Errors: ES_ERR_INVALID_ARG (NULL, generations < 1, an empty generation),

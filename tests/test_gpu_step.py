@@ -256,6 +256,33 @@ def test_replay_is_bit_identical_to_sequential_updates(es, dtype):
     plan_b.close()
 
 
+def test_replay_of_many_small_generations_is_bit_identical(es):
+    # 600 generations of 1..3 seeds: they are fused, so the limit of 256
+    # generations per pass is reached; a few larger generations in between
+    # take passes of their own.
+    numels = [8193, 4096 * 3 + 5]
+    a = make_params("bf16", numels, seed=18)
+    b = [t.clone() for t in a]
+    plan_a, _ = build_plan(es, a)
+    plan_b, _ = build_plan(es, b)
+    rng = np.random.default_rng(19)
+    counts = rng.integers(1, 4, size=600)
+    counts[[100, 101, 400]] = [5, 12, 4]
+    total = int(counts.sum())
+    seeds = rng.integers(0, 2**63, size=total, dtype=np.uint64)
+    coeffs = (1e-3 * rng.standard_normal(total)).astype(np.float32)
+    off = 0
+    for c in counts:
+        es.es_update(plan_a, seeds[off:off + c], coeffs[off:off + c])
+        off += c
+    es.es_replay(plan_b, seeds, coeffs, counts)
+    torch.cuda.synchronize()
+    for x, y in zip(a, b):
+        assert torch.equal(_int_view(x), _int_view(y))
+    plan_a.close()
+    plan_b.close()
+
+
 @pytest.mark.parametrize("dtype", ["bf16", "f32"])
 def test_update_perturb_is_bit_identical_to_the_two_calls(es, oracle, dtype):
     a = make_params(dtype, RAGGED, seed=10)
