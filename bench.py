@@ -61,6 +61,11 @@ def parse():
                    help="instead of the step: K logged generations applied by one es_replay "
                         "against K es_update calls (default workload qwen4b)")
     p.add_argument("--generations", type=int, default=16, help="K of --replay")
+    p.add_argument("--generator", action="store_true",
+                   help="instead of the step: the noise generator alone through es_noise_fill "
+                        "(2^31 Gaussians per launch) and es_noise_bits")
+    p.add_argument("--gen-log2", type=int, default=31,
+                   help="--generator: 2^k Gaussians per es_noise_fill launch")
     p.add_argument("--antithetic", action="store_true",
                    help="instead of the step: a generation of N/2 antithetic pairs (the +/- "
                         "flip as one es_restore_perturb on one seed)")
@@ -684,6 +689,58 @@ def run_replay(args, rank, world, dist):
         print(json.dumps(out), flush=True)
 
 
+def run_generator(args, rank, world, dist):
+    """The generator alone: es_noise_fill materialises 2^k Gaussians of one
+    seed (4 bytes written per Gaussian, below what HBM sustains at the
+    generator's rate, so the launch is generator-bound), and es_noise_bits
+    writes the raw Philox words of as many elements (HBM-bound)."""
+    import torch
+    from paper_2608_17310_gb300 import build, esopt as es
+
+    build.build_library()
+    dev_index = torch.cuda.current_device()
+    torch.cuda.init()
+    stream = torch.cuda.current_stream()
+    sh = stream.cuda_stream
+    n = 1 << args.gen_log2
+    eps = torch.empty(n, dtype=torch.float32, device="cuda")
+    nblocks = n >> 2
+    words = torch.empty(4 * nblocks, dtype=torch.int32, device="cuda")
+    pk = alu_peaks(torch, dev_index)
+    seed = [1000]
+
+    def fill():
+        es.es_noise_fill(seed[0], 0, n, eps, sh)
+        seed[0] += 1
+
+    def bits():
+        es.es_noise_bits(seed[0], 0, nblocks, words, sh)
+        seed[0] += 1
+
+    with ClockSampler(dev_index) as clk:
+        for _ in range(args.warmup):
+            fill()
+            bits()
+        ms_fill = _timed(torch, stream, fill, args.steps)
+        ms_bits = _timed(torch, stream, bits, args.steps)
+    fill_rates = _rates(n, 1, 4 * n, ms_fill, pk)
+    bits_gbs = 16 * nblocks / (ms_bits / 1e3) / 1e9
+    out = {"mode": "generator", "metric": "Gaussians/s of the noise generator (es_noise_fill)",
+           "unit": "Gaussians/s", "value": fill_rates["gauss_per_s"], "n_gpus": 1,
+           "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_fill,
+           "higher_is_better": True, "dtype": "f32", "data": "synthetic",
+           "config": {"gaussians_per_launch": n,
+                      "output": "fp32, %.2f GB (%s than L2)" % (4 * n / 1e9,
+                                                                "larger" if 4 * n > L2_BYTES else "smaller"),
+                      "philox_blocks_per_bits_launch": nblocks},
+           "noise_fill": fill_rates,
+           "noise_bits": {"ms": ms_bits, "words_per_s": 4 * nblocks / (ms_bits / 1e3),
+                          "gbs": bits_gbs, "hbm_frac": bits_gbs / pk[5]},
+           "gpu_launches": 2 * args.steps, "clocks": clk.summary()}
+    if rank == 0:
+        print(json.dumps(out), flush=True)
+
+
 def run_antithetic(args, rank, world, dist):
     """A generation of N/2 antithetic pairs, steady state: each pair's flip from
     +sigma eps_i to -sigma eps_i is one es_restore_perturb on one seed (noise
@@ -1091,6 +1148,8 @@ def main():
             run_replay(args, rank, world, dist)
         elif args.antithetic:
             run_antithetic(args, rank, world, dist)
+        elif args.generator:
+            run_generator(args, rank, world, dist)
         else:
             run_ours(args, rank, world, dist)
     finally:

@@ -497,6 +497,42 @@ noise_fill_kernel(uint64_t index_base, uint64_t n, PhiloxKey key, float* __restr
   }
 }
 
+// es_noise_fill when `out` is 16-byte aligned and index_base % 4 == 0:
+// out4[b] = eps[4 (j_first + b) .. 4 (j_first + b) + 3] for b < nblocks. Tiles
+// of 256 threads x kVecsPerThread blocks, each 16-byte store coalesced across
+// the warp; the Philox constants of the blocks' high word are hoisted per tile
+// when the tile stays within one 2^32-block range. The pair transform is the
+// packed form (bit-identical to box_muller).
+template <bool kUniformHi>
+__device__ __forceinline__ void noise_fill_tile(uint64_t j_first, uint64_t b0, uint64_t nblocks,
+                                                PhiloxKey key, float4* __restrict__ out) {
+  const auto gen = make_gen<kUniformHi>(key, static_cast<uint32_t>((j_first + b0) >> 32));
+#pragma unroll
+  for (int q = 0; q < kVecsPerThread; ++q) {
+    const uint64_t b = b0 + static_cast<uint64_t>(q * kBlockThreads + threadIdx.x);
+    if (b < nblocks) {
+      const Polar2 p = polar2(gen.block(j_first + b));
+      const float2 lo = __fmul2_rn(make_float2(-p.r.x, -p.r.x), make_float2(p.c.x, p.s.x));
+      const float2 hi = __fmul2_rn(make_float2(-p.r.y, -p.r.y), make_float2(p.c.y, p.s.y));
+      out[b] = make_float4(lo.x, lo.y, hi.x, hi.y);
+    }
+  }
+}
+
+__global__ void __launch_bounds__(kBlockThreads)
+noise_fill_vec_kernel(uint64_t j_first, uint64_t nblocks, PhiloxKey key, float4* __restrict__ out) {
+  constexpr uint64_t kTileBlocks = static_cast<uint64_t>(kBlockThreads) * kVecsPerThread;
+  const uint64_t tiles = (nblocks + kTileBlocks - 1) / kTileBlocks;
+  for (uint64_t tile = blockIdx.x; tile < tiles; tile += gridDim.x) {
+    const uint64_t b0 = tile * kTileBlocks;
+    const uint64_t last = (b0 + kTileBlocks < nblocks ? b0 + kTileBlocks : nblocks) - 1;
+    if (((j_first + b0) >> 32) == ((j_first + last) >> 32))
+      noise_fill_tile<true>(j_first, b0, nblocks, key, out);
+    else
+      noise_fill_tile<false>(j_first, b0, nblocks, key, out);
+  }
+}
+
 // out[4t .. 4t+3] = Philox words of block block_base + t. Even and odd blocks
 // go through the two implementations of the rounds (general, and with the
 // per-tile constants of philox_tile); they give identical words, and this lets
@@ -605,10 +641,25 @@ cudaError_t launch_box_muller(const uint32_t* words, uint64_t npairs, float* out
 
 cudaError_t launch_noise_fill(uint64_t seed, uint64_t index_base, uint64_t n, float* out,
                               cudaStream_t stream) {
+  const PhiloxKey key = philox_key(seed);
+  // Aligned case: whole Philox blocks as 16-byte stores; the n % 4 elements
+  // left over go through the general kernel below.
+  if (reinterpret_cast<uintptr_t>(out) % 16 == 0 && index_base % 4 == 0 && n >= 4) {
+    const uint64_t full = n / 4;
+    constexpr uint64_t kTileBlocks = static_cast<uint64_t>(kBlockThreads) * kVecsPerThread;
+    const int grid = persistent_grid(noise_fill_vec_kernel, (full + kTileBlocks - 1) / kTileBlocks);
+    noise_fill_vec_kernel<<<grid, kBlockThreads, 0, stream>>>(index_base / 4, full, key,
+                                                              reinterpret_cast<float4*>(out));
+    const cudaError_t err = cudaGetLastError();
+    if (err != cudaSuccess || n % 4 == 0) return err;
+    index_base += 4 * full;
+    out += 4 * full;
+    n %= 4;
+  }
   const uint64_t nblocks = ((index_base + n - 1) >> 2) - (index_base >> 2) + 1;
   const uint64_t ctas = (nblocks + kBlockThreads - 1) / kBlockThreads;
   const int grid = persistent_grid(noise_fill_kernel, ctas);
-  noise_fill_kernel<<<grid, kBlockThreads, 0, stream>>>(index_base, n, philox_key(seed), out);
+  noise_fill_kernel<<<grid, kBlockThreads, 0, stream>>>(index_base, n, key, out);
   return cudaGetLastError();
 }
 

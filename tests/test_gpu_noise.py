@@ -81,3 +81,27 @@ def test_noise_is_bit_identical_across_calls_and_streams(es):
         es.es_noise_fill(5, 64, b.numel(), b, stream=s)
     torch.cuda.synchronize()
     assert torch.equal(a.view(torch.int32), b.view(torch.int32))
+
+
+def test_noise_fill_aligned_path_equals_box_muller_of_the_words(es):
+    # With an aligned output and index base, whole Philox blocks take the
+    # 16-byte store path (packed transform); they must equal, bit for bit,
+    # es_box_muller (scalar transform) applied to the same es_noise_bits words.
+    # Ranges: plain, crossing the 2^32-block boundary, far out, ragged tails.
+    seed = 424242
+    for block_base, nb, extra in ((0, 4096 + 3, 0), (2**32 - 700, 1500, 3), (2**40 + 12, 999, 2)):
+        words = torch.empty(4 * nb, dtype=torch.int32, device="cuda")
+        es.es_noise_bits(seed, block_base, nb, words)
+        bm = torch.empty(4 * nb, dtype=torch.float32, device="cuda")
+        es.es_box_muller(words, 2 * nb, bm)
+        torch.cuda.synchronize()
+        got = _fill(es, seed, 4 * block_base, 4 * nb + extra)
+        assert np.array_equal(got[:4 * nb].view(np.uint32), bm.cpu().numpy().view(np.uint32))
+
+
+def test_noise_fill_large_aligned_range_matches_oracle(es, oracle):
+    # 1,000,002 Gaussians from g = 2^34 - 16384: the aligned path across the
+    # j = 2^32 block boundary, then a 2-element tail.
+    base, n = 2**34 - 16384, 1_000_002
+    got = _fill(es, 77, base, n)
+    assert_eps_close(got, oracle.noise_fill(77, base, n), "aligned n=1e6+2")
