@@ -13,10 +13,10 @@
  *   c_i   <- alpha * Rhat_i / G  (§3; optionally / sigma)  es_update_coeffs
  *   theta <- theta + sum_i c_i * eps_{s_i}    (one pass)    es_update
  *
- * The noise eps_s is never stored: it is regenerated from the seed whenever it
- * is needed: per member only its integer seed is kept (§3; App. D.6). The
- * paper does not name a generator; this library fixes it as follows, for every
- * entry point:
+ * The noise eps_s is never stored. Per member only its integer seed is kept,
+ * and the noise is regenerated from it whenever it is needed (§3; App. D.6).
+ * The paper does not name a generator; this library fixes it as follows, for
+ * every entry point:
  *
  *   block j = floor(g / 4) of global parameter index g,
  *   Philox4x32-10 (Salmon et al., SC'11) with key = (seed_lo32, seed_hi32) and
