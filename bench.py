@@ -883,90 +883,115 @@ def e2e_fits(torch, nbytes: int, dist) -> bool:
     return bool(t.item())
 
 
-def run_e2e(args, torch, es, plan, flat, params, wl, n, esize, sigma_at, s_handle, dist, world,
-            fused, groups=8, nstreams=4):
-    """Same generation with the parameter set in pinned host memory: every step
-    copies it to the device, runs the generation through the C ABI and copies it
-    back. The tensors are split into `groups` contiguous groups with a plan
+class E2ELoop:
+    """The generation with the parameter set in pinned host memory: every step
+    copies it to the device, runs the generation through the C ABI and copies
+    it back. The tensors are split into `groups` contiguous groups with a plan
     each, so that each group's first pass starts when its copy has landed and
     its copy back starts when its last pass is done (the middle passes use the
     whole plan). The results are those of the unsplit calls: every call is
-    elementwise."""
+    elementwise (tested)."""
+
+    def __init__(self, torch, es, plan, flat, params, wl, n, esize, sigma_at, s_handle, fused,
+                 groups=8, nstreams=4):
+        self.torch, self.es, self.plan, self.flat = torch, es, plan, flat
+        self.wl, self.n, self.sigma_at, self.s_handle, self.fused = wl, n, sigma_at, s_handle, fused
+        self.nstreams = nstreams
+        self.pinned = PinnedHostBuffer(torch, flat)
+        self.host = self.pinned.tensor
+        self.host.copy_(flat)
+        self.stream = torch.cuda.current_stream()
+        self.copy_streams = [torch.cuda.Stream() for _ in range(nstreams)]
+        self.bytes_per_copy = flat.numel() * esize
+        # contiguous groups of tensors with about equal bytes
+        ends, acc, target = [], 0, sum(p.numel() for p in params) / groups
+        for k, p in enumerate(params):
+            acc += p.numel()
+            if acc >= target * (len(ends) + 1) or k == len(params) - 1:
+                ends.append(k + 1)
+        self.spans, start = [], 0
+        segs_all = es.segments_from_tensors(params)
+        for e in ends:
+            lo = params[start].data_ptr() - flat.data_ptr()
+            hi = params[e - 1].data_ptr() - flat.data_ptr() + params[e - 1].numel() * esize
+            self.spans.append((lo // esize, hi // esize,
+                               es.es_plan_create(segs_all[start:e], plan.dtype, params[start:e])))
+            start = e
+
+    def step(self, t, record=None):
+        torch, es, plan, flat, host = self.torch, self.es, self.plan, self.flat, self.host
+        wl, n, sh, stream = self.wl, self.n, self.s_handle, self.stream
+        seeds, rewards = generation_inputs(wl, t, n)
+        sigma, sigma_next = self.sigma_at(t), self.sigma_at(t + 1)
+        ev = [torch.cuda.Event(enable_timing=True) for _ in range(4)]
+        ev[0].record(stream)
+        # in: copy each group, then its first pass of the generation
+        for g, (a, b, gplan) in enumerate(self.spans):
+            cs = self.copy_streams[g % self.nstreams]
+            if g < self.nstreams:
+                cs.wait_stream(stream)
+            with torch.cuda.stream(cs):
+                flat[a:b].copy_(host[a:b], non_blocking=True)
+            stream.wait_stream(cs)
+            if not self.fused:
+                es.es_perturb(gplan, int(seeds[0]), sigma, sh)
+            elif n > 1:
+                es.es_restore_perturb(gplan, int(seeds[0]), sigma, int(seeds[1]), sigma, sh)
+            else:
+                es.es_restore(gplan, int(seeds[0]), sigma, sh)
+        ev[1].record(stream)
+        # middle of the generation on the whole plan
+        if self.fused:
+            for i in range(2, n):
+                es.es_restore_perturb(plan, int(seeds[i - 1]), sigma, int(seeds[i]), sigma, sh)
+            if n > 1:
+                es.es_restore(plan, int(seeds[n - 1]), sigma, sh)
+        else:
+            es.es_restore(plan, int(seeds[0]), sigma, sh)
+            for i in range(1, n):
+                es.es_perturb(plan, int(seeds[i]), sigma, sh)
+                es.es_restore(plan, int(seeds[i]), sigma, sh)
+        coeffs = es.es_update_coeffs(es.es_normalize_rewards(rewards, 1e-8), wl.alpha, sigma,
+                                     es.ES_SCALE_PAPER)
+        first_next = int(generation_inputs(wl, t + 1, n)[0][0])
+        ev[2].record(stream)
+        # out: last pass per group, then copy it back
+        for g, (a, b, gplan) in enumerate(self.spans):
+            if self.fused:
+                es.es_update_perturb(gplan, seeds, coeffs, first_next, sigma_next, sh)
+            else:
+                es.es_update(gplan, seeds, coeffs, sh)
+            cs = self.copy_streams[g % self.nstreams]
+            cs.wait_stream(stream)
+            with torch.cuda.stream(cs):
+                host[a:b].copy_(flat[a:b], non_blocking=True)
+        for cs in self.copy_streams:
+            stream.wait_stream(cs)
+        ev[3].record(stream)
+        if record is not None:
+            record.append(ev)
+
+    def close(self):
+        for _, _, gplan in self.spans:
+            gplan.close()
+        self.spans = []
+        self.host = None
+        self.pinned.close()
+
+
+def run_e2e(args, torch, es, plan, flat, params, wl, n, esize, sigma_at, s_handle, dist, world,
+            fused, groups=8, nstreams=4):
+    """e2e leg of the JSON line: E2ELoop timed over args.e2e_steps generations."""
     nbytes = flat.numel() * esize
     if not e2e_fits(torch, nbytes, dist):
         local = int(os.environ.get("LOCAL_WORLD_SIZE", "1"))
         return {"value": None, "unit": UNIT, "unavailable":
                 f"host memory: {local} ranks x {nbytes / 1e9:.1f} GB page-locked would exceed "
                 f"2/3 of the {host_memory_available() / 1e9:.0f} GB available"}
-    pinned = PinnedHostBuffer(torch, flat)
-    host = pinned.tensor
-    host.copy_(flat)
-    stream = torch.cuda.current_stream()
-    copy_streams = [torch.cuda.Stream() for _ in range(nstreams)]
-    bytes_per_copy = flat.numel() * esize
-    # contiguous groups of tensors with about equal bytes
-    ends, acc, target = [], 0, sum(p.numel() for p in params) / groups
-    for k, p in enumerate(params):
-        acc += p.numel()
-        if acc >= target * (len(ends) + 1) or k == len(params) - 1:
-            ends.append(k + 1)
-    spans, start = [], 0
-    for e in ends:
-        lo = params[start].data_ptr() - flat.data_ptr()
-        hi = params[e - 1].data_ptr() - flat.data_ptr() + params[e - 1].numel() * esize
-        segs = es.segments_from_tensors(params)[start:e]
-        spans.append((lo // esize, hi // esize, es.es_plan_create(segs, plan.dtype, params[start:e])))
-        start = e
-
-    def one(t, record):
-        seeds, rewards = generation_inputs(wl, t, n)
-        sigma, sigma_next = sigma_at(t), sigma_at(t + 1)
-        ev = [torch.cuda.Event(enable_timing=True) for _ in range(4)]
-        ev[0].record(stream)
-        # in: copy each group, then its first pass of the generation
-        for g, (a, b, gplan) in enumerate(spans):
-            cs = copy_streams[g % nstreams]
-            if g < nstreams:
-                cs.wait_stream(stream)
-            with torch.cuda.stream(cs):
-                flat[a:b].copy_(host[a:b], non_blocking=True)
-            stream.wait_stream(cs)
-            if fused:
-                es.es_restore_perturb(gplan, int(seeds[0]), sigma, int(seeds[1]), sigma, s_handle)
-            else:
-                es.es_perturb(gplan, int(seeds[0]), sigma, s_handle)
-        ev[1].record(stream)
-        # middle of the generation on the whole plan
-        if fused:
-            for i in range(2, n):
-                es.es_restore_perturb(plan, int(seeds[i - 1]), sigma, int(seeds[i]), sigma, s_handle)
-            es.es_restore(plan, int(seeds[n - 1]), sigma, s_handle)
-        else:
-            es.es_restore(plan, int(seeds[0]), sigma, s_handle)
-            for i in range(1, n):
-                es.es_perturb(plan, int(seeds[i]), sigma, s_handle)
-                es.es_restore(plan, int(seeds[i]), sigma, s_handle)
-        coeffs = es.es_update_coeffs(es.es_normalize_rewards(rewards, 1e-8), wl.alpha, sigma,
-                                     es.ES_SCALE_PAPER)
-        first_next = int(generation_inputs(wl, t + 1, n)[0][0])
-        ev[2].record(stream)
-        # out: last pass per group, then copy it back
-        for g, (a, b, gplan) in enumerate(spans):
-            if fused:
-                es.es_update_perturb(gplan, seeds, coeffs, first_next, sigma_next, s_handle)
-            else:
-                es.es_update(gplan, seeds, coeffs, s_handle)
-            cs = copy_streams[g % nstreams]
-            cs.wait_stream(stream)
-            with torch.cuda.stream(cs):
-                host[a:b].copy_(flat[a:b], non_blocking=True)
-        for cs in copy_streams:
-            stream.wait_stream(cs)
-        ev[3].record(stream)
-        if record is not None:
-            record.append(ev)
-
-    one(0, None)
+    loop = E2ELoop(torch, es, plan, flat, params, wl, n, esize, sigma_at, s_handle, fused,
+                   groups, nstreams)
+    stream = loop.stream
+    loop.step(0)
     torch.cuda.synchronize()
     barrier(dist)
     evs = []
@@ -974,7 +999,7 @@ def run_e2e(args, torch, es, plan, flat, params, wl, n, esize, sigma_at, s_handl
     e1 = torch.cuda.Event(enable_timing=True)
     e0.record(stream)
     for k in range(args.e2e_steps):
-        one(args.warmup + k, evs)
+        loop.step(args.warmup + k, evs)
     e1.record(stream)
     torch.cuda.synchronize()
     ms = max_over_ranks(e0.elapsed_time(e1), dist)
@@ -983,17 +1008,15 @@ def run_e2e(args, torch, es, plan, flat, params, wl, n, esize, sigma_at, s_handl
         for name, a, b in (("copy_in_and_first_pass", 0, 1), ("middle_passes", 1, 2),
                            ("last_pass_and_copy_out", 2, 3)):
             phases[name] += ev[a].elapsed_time(ev[b]) / len(evs)
-    for _, _, gplan in spans:
-        gplan.close()
+    kind, ngroups, bytes_per_copy = loop.pinned.kind, len(loop.spans), loop.bytes_per_copy
+    loop.close()
     P = sum(p.numel() for p in params)
-    del host
-    pinned.close()
     return {"value": world * P * n * args.e2e_steps / (ms / 1e3), "unit": UNIT,
             "steps": args.e2e_steps, "ms_per_step": ms / args.e2e_steps,
             "h2d_bytes_per_step": bytes_per_copy, "d2h_bytes_per_step": bytes_per_copy,
             "phase_ms": phases,
-            "layout": f"one page-locked host buffer ({pinned.kind}) and one device buffer "
-                      f"holding every tensor; {len(spans)} groups with a plan each, copies over "
+            "layout": f"one page-locked host buffer ({kind}) and one device buffer "
+                      f"holding every tensor; {ngroups} groups with a plan each, copies over "
                       f"{nstreams} streams overlapping the first and last pass of each generation"}
 
 
