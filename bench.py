@@ -903,12 +903,25 @@ class E2ELoop:
         self.stream = torch.cuda.current_stream()
         self.copy_streams = [torch.cuda.Stream() for _ in range(nstreams)]
         self.bytes_per_copy = flat.numel() * esize
-        # contiguous groups of tensors with about equal bytes
-        ends, acc, target = [], 0, sum(p.numel() for p in params) / groups
-        for k, p in enumerate(params):
-            acc += p.numel()
-            if acc >= target * (len(ends) + 1) or k == len(params) - 1:
+        # contiguous groups of tensors: the last group holds the trailing
+        # tensors up to 1/32 of the parameters (at least one tensor), since its
+        # copy back after the last update and its first pass after the last
+        # copy in are the parts no other work hides; the rest is split into
+        # groups - 1 groups of about equal size
+        sizes = [p.numel() for p in params]
+        total = sum(sizes)
+        tail, acc = len(sizes), 0
+        while tail > 1 and (acc == 0 or acc + sizes[tail - 1] <= total / 32):
+            tail -= 1
+            acc += sizes[tail]
+        ends, acc = [], 0
+        head = sum(sizes[:tail])
+        for k in range(tail):
+            acc += sizes[k]
+            if acc >= head * (len(ends) + 1) / max(groups - 1, 1) or k == tail - 1:
                 ends.append(k + 1)
+        if tail < len(sizes):
+            ends.append(len(sizes))
         self.spans, start = [], 0
         segs_all = es.segments_from_tensors(params)
         for e in ends:
