@@ -833,6 +833,7 @@ class PinnedHostBuffer:
         self.torch = torch
         self.addr = None
         nbytes = like.numel() * like.element_size()
+        self.nbytes = nbytes
         try:
             self.map = mmap.mmap(-1, nbytes, flags=mmap.MAP_PRIVATE | mmap.MAP_ANONYMOUS)
             addr = ctypes.addressof(ctypes.c_char.from_buffer(self.map))
@@ -849,6 +850,26 @@ class PinnedHostBuffer:
             self.map = None
             self.tensor = torch.empty(like.shape, dtype=like.dtype, pin_memory=True)
             self.kind = "torch pin_memory"
+
+    def hugepage_fraction(self):
+        """Share of the buffer backed by transparent huge pages (None if the
+        buffer is torch's, or /proc/self/smaps cannot be read)."""
+        if self.addr is None:
+            return None
+        lo, hi = self.addr, self.addr + self.nbytes
+        huge, cur = 0, False
+        try:
+            with open("/proc/self/smaps") as f:
+                for line in f:
+                    head = line.split()[0]
+                    if "-" in head and not head.endswith(":"):
+                        a, b = (int(x, 16) for x in head.split("-"))
+                        cur = a < hi and b > lo
+                    elif cur and head == "AnonHugePages:":
+                        huge += int(line.split()[1]) * 1024
+        except (OSError, ValueError):
+            return None
+        return min(1.0, huge / self.nbytes)
 
     def close(self):
         if self.addr is not None:
@@ -1022,12 +1043,13 @@ def run_e2e(args, torch, es, plan, flat, params, wl, n, esize, sigma_at, s_handl
                            ("last_pass_and_copy_out", 2, 3)):
             phases[name] += ev[a].elapsed_time(ev[b]) / len(evs)
     kind, ngroups, bytes_per_copy = loop.pinned.kind, len(loop.spans), loop.bytes_per_copy
+    huge = loop.pinned.hugepage_fraction()
     loop.close()
     P = sum(p.numel() for p in params)
     return {"value": world * P * n * args.e2e_steps / (ms / 1e3), "unit": UNIT,
             "steps": args.e2e_steps, "ms_per_step": ms / args.e2e_steps,
             "h2d_bytes_per_step": bytes_per_copy, "d2h_bytes_per_step": bytes_per_copy,
-            "phase_ms": phases,
+            "phase_ms": phases, "host_hugepage_fraction": huge,
             "layout": f"one page-locked host buffer ({kind}) and one device buffer "
                       f"holding every tensor; {ngroups} groups with a plan each, copies over "
                       f"{nstreams} streams overlapping the first and last pass of each generation"}

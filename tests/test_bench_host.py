@@ -50,3 +50,18 @@ def test_pipe_occupancy_file_is_keyed_by_the_current_code():
     if all(r[3] == bench.kernel_code_digest() for r in rows):
         assert occ is not None and 90.0 < occ["sum_pct"] < 115.0
     assert bench.pipe_occupancy("restore") is None
+
+
+def test_hugepage_fraction_of_an_anonymous_mapping_is_a_fraction():
+    import ctypes
+    import mmap
+    import numpy as np
+    buf = bench.PinnedHostBuffer.__new__(bench.PinnedHostBuffer)
+    buf.nbytes = 16 << 20
+    m = mmap.mmap(-1, buf.nbytes, flags=mmap.MAP_PRIVATE | mmap.MAP_ANONYMOUS)
+    buf.addr = ctypes.addressof(ctypes.c_char.from_buffer(m))
+    np.frombuffer(m, dtype=np.uint8)[::4096] = 1
+    frac = buf.hugepage_fraction()
+    assert frac is None or 0.0 <= frac <= 1.0
+    buf.addr = None
+    assert buf.hugepage_fraction() is None
