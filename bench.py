@@ -824,14 +824,16 @@ class PinnedHostBuffer:
     transparent huge pages requested (madvise), registered with
     cudaHostRegister. On the GB300 machines huge-page-backed buffers copy at a
     steady 211 GB/s (H2D) / 193 GB/s (D2H); cudaHostAlloc'd memory varied
-    between 100 and 204 GB/s from run to run. Falls back to torch's pinned
-    allocator if registration fails."""
+    between 100 and 204 GB/s from run to run, and a buffer with 11 % of its
+    pages left at base size made the e2e step 2.2x slower. Falls back to
+    torch's pinned allocator if registration fails."""
 
     def __init__(self, torch, like):
         import ctypes
         import mmap
         self.torch = torch
         self.addr = None
+        self.hugepages_at_fault = None
         nbytes = like.numel() * like.element_size()
         self.nbytes = nbytes
         try:
@@ -840,7 +842,14 @@ class PinnedHostBuffer:
             libc = ctypes.CDLL(None)
             libc.madvise(ctypes.c_void_p(addr), ctypes.c_size_t(nbytes), 14)  # MADV_HUGEPAGE
             arr = np.frombuffer(self.map, dtype=np.uint8)
-            arr[::4096] = 0   # fault the pages in before registering them
+            # Fault the pages in before registering them, with a non-zero byte
+            # in every 4 KB: the kernel may split a huge page whose subpages are
+            # all zero to reclaim them, and a buffer partly on base pages copies
+            # several times slower.
+            arr[::4096] = 1
+            self.addr = addr
+            self.hugepages_at_fault = self.hugepage_fraction()
+            self.addr = None
             if int(torch.cuda.cudart().cudaHostRegister(addr, nbytes, 0)) != 0:
                 raise OSError("cudaHostRegister failed")
             self.addr = addr
@@ -959,14 +968,20 @@ class E2ELoop:
         sigma, sigma_next = self.sigma_at(t), self.sigma_at(t + 1)
         ev = [torch.cuda.Event(enable_timing=True) for _ in range(4)]
         ev[0].record(stream)
-        # in: copy each group, then its first pass of the generation
-        for g, (a, b, gplan) in enumerate(self.spans):
+        # in: every copy waits only for the previous step; each group's first
+        # pass waits only for its own copy
+        for cs in self.copy_streams:
+            cs.wait_stream(stream)
+        landed = []
+        for g, (a, b, _) in enumerate(self.spans):
             cs = self.copy_streams[g % self.nstreams]
-            if g < self.nstreams:
-                cs.wait_stream(stream)
             with torch.cuda.stream(cs):
                 flat[a:b].copy_(host[a:b], non_blocking=True)
-            stream.wait_stream(cs)
+                done = torch.cuda.Event()
+                done.record(cs)
+            landed.append(done)
+        for (a, b, gplan), done in zip(self.spans, landed):
+            stream.wait_event(done)
             if not self.fused:
                 es.es_perturb(gplan, int(seeds[0]), sigma, sh)
             elif n > 1:
@@ -1044,12 +1059,14 @@ def run_e2e(args, torch, es, plan, flat, params, wl, n, esize, sigma_at, s_handl
             phases[name] += ev[a].elapsed_time(ev[b]) / len(evs)
     kind, ngroups, bytes_per_copy = loop.pinned.kind, len(loop.spans), loop.bytes_per_copy
     huge = loop.pinned.hugepage_fraction()
+    hp_fault = loop.pinned.hugepages_at_fault
     loop.close()
     P = sum(p.numel() for p in params)
     return {"value": world * P * n * args.e2e_steps / (ms / 1e3), "unit": UNIT,
             "steps": args.e2e_steps, "ms_per_step": ms / args.e2e_steps,
             "h2d_bytes_per_step": bytes_per_copy, "d2h_bytes_per_step": bytes_per_copy,
             "phase_ms": phases, "host_hugepage_fraction": huge,
+            "host_hugepage_fraction_at_allocation": hp_fault,
             "layout": f"one page-locked host buffer ({kind}) and one device buffer "
                       f"holding every tensor; {ngroups} groups with a plan each, copies over "
                       f"{nstreams} streams overlapping the first and last pass of each generation"}
