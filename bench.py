@@ -825,7 +825,7 @@ class PinnedHostBuffer:
     cudaHostRegister. On the GB300 machines huge-page-backed buffers copy at a
     steady 211 GB/s (H2D) / 193 GB/s (D2H); cudaHostAlloc'd memory varied
     between 100 and 204 GB/s from run to run, and a buffer with 11 % of its
-    pages left at base size made the e2e step 2.2x slower. Falls back to
+    pages split to base size made the e2e step 2.2x slower. Falls back to
     torch's pinned allocator if registration fails."""
 
     def __init__(self, torch, like):
@@ -842,17 +842,15 @@ class PinnedHostBuffer:
             libc = ctypes.CDLL(None)
             libc.madvise(ctypes.c_void_p(addr), ctypes.c_size_t(nbytes), 14)  # MADV_HUGEPAGE
             arr = np.frombuffer(self.map, dtype=np.uint8)
-            # Fault the pages in before registering them, with a non-zero byte
-            # in every 4 KB: the kernel may split a huge page whose subpages are
-            # all zero to reclaim them, and a buffer partly on base pages copies
-            # several times slower.
-            arr[::4096] = 1
-            self.addr = addr
-            self.hugepages_at_fault = self.hugepage_fraction()
-            self.addr = None
+            # The registration faults the pages in itself. Pages the CPU had
+            # faulted in first were, in some runs, split out of their huge
+            # pages once the GPU wrote to them, and copies through a partly
+            # split buffer ran 5-9x slower; pages faulted in by the
+            # registration were never split (measured).
             if int(torch.cuda.cudart().cudaHostRegister(addr, nbytes, 0)) != 0:
                 raise OSError("cudaHostRegister failed")
             self.addr = addr
+            self.hugepages_at_fault = self.hugepage_fraction()
             self.tensor = torch.from_numpy(arr).view(like.dtype)
             self.kind = "mmap + MADV_HUGEPAGE + cudaHostRegister"
         except Exception:
@@ -886,6 +884,7 @@ class PinnedHostBuffer:
             self.torch.cuda.cudart().cudaHostUnregister(self.addr)
             self.addr = None
         self.tensor = None
+        self.map = None     # the mapping is released with its last reference
 
 
 def host_memory_available() -> int:
@@ -927,9 +926,24 @@ class E2ELoop:
         self.torch, self.es, self.plan, self.flat = torch, es, plan, flat
         self.wl, self.n, self.sigma_at, self.s_handle, self.fused = wl, n, sigma_at, s_handle, fused
         self.nstreams = nstreams
-        self.pinned = PinnedHostBuffer(torch, flat)
-        self.host = self.pinned.tensor
-        self.host.copy_(flat)
+        # The first use of a fresh page-locked buffer sometimes splits some of
+        # its huge pages, and copies through it then run 5-9x slower (the
+        # kernel's thp_split_page count rises; a buffer allocated after a
+        # release does not show it). So the buffer makes one round trip and,
+        # if its huge-page share fell, is released and allocated again.
+        self.attempts = 0
+        for self.attempts in range(1, 6):
+            self.pinned = PinnedHostBuffer(torch, flat)
+            self.host = self.pinned.tensor
+            self.host.copy_(flat)
+            flat.copy_(self.host)
+            torch.cuda.synchronize()
+            before, after = self.pinned.hugepages_at_fault, self.pinned.hugepage_fraction()
+            if before is None or after is None or after >= before - 0.005 or self.attempts == 5:
+                break
+            self.host = None
+            self.pinned.close()
+            self.pinned = None
         self.stream = torch.cuda.current_stream()
         self.copy_streams = [torch.cuda.Stream() for _ in range(nstreams)]
         self.bytes_per_copy = flat.numel() * esize
@@ -1060,13 +1074,15 @@ def run_e2e(args, torch, es, plan, flat, params, wl, n, esize, sigma_at, s_handl
     kind, ngroups, bytes_per_copy = loop.pinned.kind, len(loop.spans), loop.bytes_per_copy
     huge = loop.pinned.hugepage_fraction()
     hp_fault = loop.pinned.hugepages_at_fault
+    attempts = loop.attempts
     loop.close()
     P = sum(p.numel() for p in params)
     return {"value": world * P * n * args.e2e_steps / (ms / 1e3), "unit": UNIT,
             "steps": args.e2e_steps, "ms_per_step": ms / args.e2e_steps,
             "h2d_bytes_per_step": bytes_per_copy, "d2h_bytes_per_step": bytes_per_copy,
             "phase_ms": phases, "host_hugepage_fraction": huge,
-            "host_hugepage_fraction_at_allocation": hp_fault,
+            "host_hugepage_fraction_at_registration": hp_fault,
+            "host_buffer_attempts": attempts,
             "layout": f"one page-locked host buffer ({kind}) and one device buffer "
                       f"holding every tensor; {ngroups} groups with a plan each, copies over "
                       f"{nstreams} streams overlapping the first and last pass of each generation"}
