@@ -9,8 +9,8 @@
   qwen27b    22,695,777,280 bf16 parameters in 579 tensors, N = 30
   sweep      the 4B set with N in {1, 2, 4, 8, 16, 32, 64, 128}
 At full size the oracle checks, for every call, the first and last 64 elements
-of every tensor plus random elements, in the launch configuration the
-benchmark times.
+of every tensor plus about 10^6 random elements, in the launch configuration
+the benchmark times.
 """
 import gc
 
@@ -204,11 +204,13 @@ def _llm_generation(es, oracle, workload, n_random, check_members, reward_kind=N
 
 
 def test_qwen4b_generation_full_size(es, oracle):
-    _llm_generation(es, oracle, "qwen4b", n_random=300, check_members=set(range(16)))
+    # 326 tensors x (3000 random + 128 edge) elements: about 10^6 sampled indices
+    _llm_generation(es, oracle, "qwen4b", n_random=3000, check_members=set(range(16)))
 
 
 def test_qwen27b_generation_full_size(es, oracle):
-    _llm_generation(es, oracle, "qwen27b", n_random=150, check_members={0, 1, 14, 29})
+    # 579 tensors x (1700 random + 128 edge) elements: about 10^6 sampled indices
+    _llm_generation(es, oracle, "qwen27b", n_random=1700, check_members={0, 1, 14, 29})
 
 
 def test_population_sweep_on_qwen4b(es, oracle):
