@@ -917,6 +917,28 @@ def e2e_fits(torch, nbytes: int, dist) -> bool:
     return bool(t.item())
 
 
+def copy_groups(sizes, groups=8):
+    """Ends (exclusive tensor indices) of the contiguous copy groups of the e2e
+    leg. The last group holds the trailing tensors up to 1/32 of the elements
+    (at least one tensor): its copy back after the last update and its first
+    pass after the last copy in are the parts no other work hides. The rest is
+    split into groups - 1 groups of about equal size."""
+    total = sum(sizes)
+    tail, acc = len(sizes), 0
+    while tail > 1 and (acc == 0 or acc + sizes[tail - 1] <= total / 32):
+        tail -= 1
+        acc += sizes[tail]
+    ends, acc = [], 0
+    head = sum(sizes[:tail])
+    for k in range(tail):
+        acc += sizes[k]
+        if acc >= head * (len(ends) + 1) / max(groups - 1, 1) or k == tail - 1:
+            ends.append(k + 1)
+    if tail < len(sizes):
+        ends.append(len(sizes))
+    return ends
+
+
 class E2ELoop:
     """The generation with the parameter set in pinned host memory: every step
     copies it to the device, runs the generation through the C ABI and copies
@@ -952,25 +974,7 @@ class E2ELoop:
         self.stream = torch.cuda.current_stream()
         self.copy_streams = [torch.cuda.Stream() for _ in range(nstreams)]
         self.bytes_per_copy = flat.numel() * esize
-        # contiguous groups of tensors: the last group holds the trailing
-        # tensors up to 1/32 of the parameters (at least one tensor), since its
-        # copy back after the last update and its first pass after the last
-        # copy in are the parts no other work hides; the rest is split into
-        # groups - 1 groups of about equal size
-        sizes = [p.numel() for p in params]
-        total = sum(sizes)
-        tail, acc = len(sizes), 0
-        while tail > 1 and (acc == 0 or acc + sizes[tail - 1] <= total / 32):
-            tail -= 1
-            acc += sizes[tail]
-        ends, acc = [], 0
-        head = sum(sizes[:tail])
-        for k in range(tail):
-            acc += sizes[k]
-            if acc >= head * (len(ends) + 1) / max(groups - 1, 1) or k == tail - 1:
-                ends.append(k + 1)
-        if tail < len(sizes):
-            ends.append(len(sizes))
+        ends = copy_groups([p.numel() for p in params], groups)
         self.spans, start = [], 0
         segs_all = es.segments_from_tensors(params)
         for e in ends:

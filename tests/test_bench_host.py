@@ -65,3 +65,16 @@ def test_hugepage_fraction_of_an_anonymous_mapping_is_a_fraction():
     assert frac is None or 0.0 <= frac <= 1.0
     buf.addr = None
     assert buf.hugepage_fraction() is None
+
+
+def test_copy_groups_cover_every_tensor_with_a_small_last_group():
+    from paper_2608_17310_gb300 import inputs as I
+    for name in ("qwen27b", "qwen4b", "qwen4b_4layer", "toy"):
+        sizes = [s.numel for s in I.shapes_for(name)]
+        ends = bench.copy_groups(sizes, 8)
+        assert ends[-1] == len(sizes) and len(ends) <= 8
+        assert all(b > a for a, b in zip([0] + ends[:-1], ends))   # non-empty, in order
+        last = sizes[(ends[-2] if len(ends) > 1 else 0):]
+        assert len(last) == 1 or sum(last) <= sum(sizes) / 32
+    assert bench.copy_groups([5], 8) == [1]
+    assert bench.copy_groups([1] * 64, 8)[-1] == 64
