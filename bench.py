@@ -838,7 +838,7 @@ class PinnedHostBuffer:
         import mmap
         self.torch = torch
         self.addr = None
-        self.hugepages_at_fault = None
+        self.hugepages_at_registration = None
         nbytes = like.numel() * like.element_size()
         self.nbytes = nbytes
         try:
@@ -855,7 +855,7 @@ class PinnedHostBuffer:
             if int(torch.cuda.cudart().cudaHostRegister(addr, nbytes, 0)) != 0:
                 raise OSError("cudaHostRegister failed")
             self.addr = addr
-            self.hugepages_at_fault = self.hugepage_fraction()
+            self.hugepages_at_registration = self.hugepage_fraction()
             self.tensor = torch.from_numpy(arr).view(like.dtype)
             self.kind = "mmap + MADV_HUGEPAGE + cudaHostRegister"
         except Exception:
@@ -965,7 +965,7 @@ class E2ELoop:
             self.host.copy_(flat)
             flat.copy_(self.host)
             torch.cuda.synchronize()
-            before, after = self.pinned.hugepages_at_fault, self.pinned.hugepage_fraction()
+            before, after = self.pinned.hugepages_at_registration, self.pinned.hugepage_fraction()
             if before is None or after is None or after >= before - 0.005 or self.attempts == 5:
                 break
             self.host = None
@@ -1082,7 +1082,7 @@ def run_e2e(args, torch, es, plan, flat, params, wl, n, esize, sigma_at, s_handl
             phases[name] += ev[a].elapsed_time(ev[b]) / len(evs)
     kind, ngroups, bytes_per_copy = loop.pinned.kind, len(loop.spans), loop.bytes_per_copy
     huge = loop.pinned.hugepage_fraction()
-    hp_fault = loop.pinned.hugepages_at_fault
+    hp_fault = loop.pinned.hugepages_at_registration
     attempts = loop.attempts
     loop.close()
     P = sum(p.numel() for p in params)
