@@ -27,7 +27,8 @@
  *     alpha/(G sigma) of App. C.1), and the antithetic fold.
  *
  * R is one rounding of the double-precision value to the storage type
- * (round-to-nearest-even for both fp32 and bf16).
+ * (round-to-nearest-even for fp32, bf16 and FP8 E4M3; E4M3 saturates at its
+ * largest finite value and is stored with a per-segment scale).
  *
  * Parity is pinned against: an independent Philox implementation (PyTorch's
  * host engine), closed forms, invariants and brute-force Monte Carlo checks in
@@ -187,6 +188,59 @@ uint16_t oracle_bf16_from_double(double x) {
 /* Round a double to binary32, ties to even (the C conversion). */
 float oracle_f32_from_double(double x) { return (float)x; }
 
+/*
+ * FP8 E4M3 storage (the quantized-weight direction the paper leaves as future
+ * work, App. A.2; only the storage grid is new, the step is unchanged). The
+ * E4M3 format of the OCP 8-bit floating-point specification: 1 sign bit, 4
+ * exponent bits with bias 7, 3 mantissa bits; exponent 0 holds the subnormals
+ * m * 2^-9; there are no infinities, exponent 15 with mantissa 7 is NaN, and
+ * the largest finite magnitude is 1.75 * 2^8 = 448.
+ *
+ * A segment stored in E4M3 carries one scale s > 0: element k has the value
+ * s * e4m3(code[k]).
+ */
+double oracle_e4m3_to_double(uint8_t c) {
+  int exponent = (c >> 3) & 0xF;
+  int mantissa = c & 0x7;
+  double v;
+  if (exponent == 0xF && mantissa == 0x7)
+    v = NAN;
+  else if (exponent == 0)
+    v = mantissa * 0x1p-9;
+  else
+    v = ldexp(1.0 + mantissa / 8.0, exponent - 7);
+  return (c & 0x80) ? -v : v;
+}
+
+/*
+ * Round a double to the nearest E4M3 value, ties to even, saturating: a
+ * magnitude beyond the largest finite value (448), infinities included,
+ * becomes 448 with its sign. NaN maps to the NaN code of the same sign.
+ */
+uint8_t oracle_e4m3_from_double(double x) {
+  uint8_t sign = signbit(x) ? 0x80u : 0x00u;
+  if (isnan(x)) return (uint8_t)(sign | 0x7Fu);
+  double a = fabs(x);
+  if (a >= 448.0) return (uint8_t)(sign | 0x7Eu);
+  double q;
+  if (a < 0x1p-6) {
+    /* subnormal range: fixed spacing 2^-9 */
+    q = rint(a * 0x1p9) * 0x1p-9;
+  } else {
+    int e;
+    frexp(a, &e); /* a = f * 2^e, f in [0.5, 1): 4 significant bits -> spacing 2^(e-4) */
+    q = ldexp(rint(ldexp(a, 4 - e)), e - 4);
+  }
+  if (q > 448.0) q = 448.0;
+  if (q == 0.0) return sign;
+  if (q < 0x1p-6) return (uint8_t)(sign | (uint8_t)(q * 0x1p9));
+  int e;
+  double f = frexp(q, &e); /* q = (2f) 2^(e-1), 2f in [1, 2) */
+  int exponent = e - 1 + 7;
+  int mantissa = (int)((2.0 * f - 1.0) * 8.0);
+  return (uint8_t)(sign | (uint8_t)(exponent << 3) | (uint8_t)mantissa);
+}
+
 /* ------------------------------------------------------------------------- */
 /* Perturb / restore / update on host arrays.                                 */
 /*                                                                           */
@@ -212,6 +266,18 @@ void oracle_axpy_noise_bf16(uint16_t* theta, const uint64_t* g, uint64_t n,
   }
 }
 
+/* Perturb / restore of an E4M3 segment with scale s: the value s * e4m3(code)
+   moves by scale * eps, and the result is stored as the nearest E4M3 code of
+   (value / s). */
+void oracle_axpy_noise_e4m3(uint8_t* codes, const uint64_t* g, uint64_t n, uint64_t seed,
+                            float scale, float seg_scale) {
+  const double s = (double)seg_scale;
+  for (uint64_t k = 0; k < n; ++k) {
+    double v = s * oracle_e4m3_to_double(codes[k]) + (double)scale * oracle_gaussian(seed, g[k]);
+    codes[k] = oracle_e4m3_from_double(v / s);
+  }
+}
+
 /*
  * theta[k] <- R(theta[k] + sum_{i=0}^{nseeds-1} coeffs[i] * eps_{seeds[i]}[g[k]]),
  * the sum taken in double in ascending i, then one rounding.
@@ -233,6 +299,20 @@ void oracle_update_bf16(uint16_t* theta, const uint64_t* g, uint64_t n,
     for (int i = 0; i < nseeds; ++i)
       sum += (double)coeffs[i] * oracle_gaussian(seeds[i], g[k]);
     theta[k] = oracle_bf16_from_double(oracle_bf16_to_double(theta[k]) + sum);
+  }
+}
+
+/* The update of an E4M3 segment with scale s: value s * e4m3(code) plus the
+   reward-weighted sum (double, ascending i), stored as the nearest E4M3 code of
+   (value / s). */
+void oracle_update_e4m3(uint8_t* codes, const uint64_t* g, uint64_t n, const uint64_t* seeds,
+                        const float* coeffs, int nseeds, float seg_scale) {
+  const double s = (double)seg_scale;
+  for (uint64_t k = 0; k < n; ++k) {
+    double sum = 0.0;
+    for (int i = 0; i < nseeds; ++i)
+      sum += (double)coeffs[i] * oracle_gaussian(seeds[i], g[k]);
+    codes[k] = oracle_e4m3_from_double((s * oracle_e4m3_to_double(codes[k]) + sum) / s);
   }
 }
 

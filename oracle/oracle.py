@@ -26,6 +26,7 @@ _lib = None
 _u64p = ctypes.POINTER(ctypes.c_uint64)
 _u32p = ctypes.POINTER(ctypes.c_uint32)
 _u16p = ctypes.POINTER(ctypes.c_uint16)
+_u8p = ctypes.POINTER(ctypes.c_uint8)
 _f32p = ctypes.POINTER(ctypes.c_float)
 _f64p = ctypes.POINTER(ctypes.c_double)
 
@@ -65,6 +66,14 @@ def lib() -> ctypes.CDLL:
             L.oracle_bf16_from_double.restype = ctypes.c_uint16
             L.oracle_f32_from_double.argtypes = [ctypes.c_double]
             L.oracle_f32_from_double.restype = ctypes.c_float
+            L.oracle_e4m3_to_double.argtypes = [ctypes.c_uint8]
+            L.oracle_e4m3_to_double.restype = ctypes.c_double
+            L.oracle_e4m3_from_double.argtypes = [ctypes.c_double]
+            L.oracle_e4m3_from_double.restype = ctypes.c_uint8
+            L.oracle_axpy_noise_e4m3.argtypes = [_u8p, _u64p, ctypes.c_uint64,
+                                                 ctypes.c_uint64, ctypes.c_float, ctypes.c_float]
+            L.oracle_update_e4m3.argtypes = [_u8p, _u64p, ctypes.c_uint64, _u64p,
+                                             _f32p, ctypes.c_int, ctypes.c_float]
             L.oracle_axpy_noise_f32.argtypes = [_f32p, _u64p, ctypes.c_uint64,
                                                 ctypes.c_uint64, ctypes.c_float]
             L.oracle_axpy_noise_bf16.argtypes = [_u16p, _u64p, ctypes.c_uint64,
@@ -161,6 +170,21 @@ def bf16_bits_to_f64(bits: np.ndarray) -> np.ndarray:
     return b.view(np.float32).astype(np.float64)
 
 
+def e4m3_to_double(c: int) -> float:
+    return lib().oracle_e4m3_to_double(c)
+
+
+def e4m3_from_double(x: float) -> int:
+    return lib().oracle_e4m3_from_double(x)
+
+
+def e4m3_codes_to_f64(codes: np.ndarray) -> np.ndarray:
+    """E4M3 codes (uint8) -> float64 values, one oracle call per code."""
+    c = np.ascontiguousarray(codes, dtype=np.uint8)
+    return np.array([lib().oracle_e4m3_to_double(int(v)) for v in c.ravel()],
+                    dtype=np.float64).reshape(c.shape)
+
+
 # --- step -----------------------------------------------------------------
 
 def _indices(g, n):
@@ -192,22 +216,50 @@ def axpy_noise_bf16(theta_bits: np.ndarray, g: np.ndarray, seed: int, scale: flo
     return t
 
 
-def perturb(theta, g, seed, sigma, dtype="f32"):
-    fn = axpy_noise_f32 if dtype == "f32" else axpy_noise_bf16
-    return fn(theta, g, seed, float(np.float32(sigma)))
+def axpy_noise_e4m3(codes: np.ndarray, g: np.ndarray, seed: int, scale: float,
+                    seg_scale: float) -> np.ndarray:
+    """E4M3 codes (uint8) of a segment with scale seg_scale: the nearest code of
+    (seg_scale * value + scale * eps_seed[g]) / seg_scale (returns a new array)."""
+    t = np.array(codes, dtype=np.uint8, copy=True, order="C")
+    g = _indices(g, t.size)
+    if t.size:
+        lib().oracle_axpy_noise_e4m3(_ptr(t, _u8p), _ptr(g, _u64p), t.size, seed,
+                                     float(np.float32(scale)), float(np.float32(seg_scale)))
+    return t
 
 
-def restore(theta, g, seed, sigma, dtype="f32"):
-    fn = axpy_noise_f32 if dtype == "f32" else axpy_noise_bf16
-    return fn(theta, g, seed, -float(np.float32(sigma)))
+def _axpy(theta, g, seed, scale, dtype, seg_scale):
+    if dtype == "f32":
+        return axpy_noise_f32(theta, g, seed, scale)
+    if dtype == "bf16":
+        return axpy_noise_bf16(theta, g, seed, scale)
+    if dtype == "e4m3":
+        return axpy_noise_e4m3(theta, g, seed, scale, seg_scale)
+    raise ValueError(f"unknown storage type {dtype}")
 
 
-def update(theta, g, seeds, coeffs, dtype="f32"):
-    """theta + sum_i coeffs[i] * eps_{seeds[i]}[g], summed in double, one rounding."""
+def perturb(theta, g, seed, sigma, dtype="f32", seg_scale=1.0):
+    return _axpy(theta, g, seed, float(np.float32(sigma)), dtype, seg_scale)
+
+
+def restore(theta, g, seed, sigma, dtype="f32", seg_scale=1.0):
+    return _axpy(theta, g, seed, -float(np.float32(sigma)), dtype, seg_scale)
+
+
+def update(theta, g, seeds, coeffs, dtype="f32", seg_scale=1.0):
+    """theta + sum_i coeffs[i] * eps_{seeds[i]}[g], summed in double, one rounding
+    (for E4M3: of the scaled value, stored back divided by seg_scale)."""
     s = np.ascontiguousarray(seeds, dtype=np.uint64)
     c = np.ascontiguousarray(coeffs, dtype=np.float32)
     if s.size != c.size:
         raise ValueError("seeds and coeffs differ in length")
+    if dtype == "e4m3":
+        t = np.array(theta, dtype=np.uint8, copy=True, order="C")
+        g = _indices(g, t.size)
+        if t.size:
+            lib().oracle_update_e4m3(_ptr(t, _u8p), _ptr(g, _u64p), t.size, _ptr(s, _u64p),
+                                     _ptr(c, _f32p), s.size, float(np.float32(seg_scale)))
+        return t
     if dtype == "f32":
         t = np.array(theta, dtype=np.float32, copy=True, order="C")
         g = _indices(g, t.size)
