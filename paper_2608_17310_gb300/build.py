@@ -1,8 +1,10 @@
-"""Builds the in-tree CUDA library ``_build/libesopt.so`` for sm_103a.
+"""Builds the in-tree CUDA library ``_build/libesopt.so`` for sm_103a, and the
+pipe-probe library ``_build/libesprobe.so`` that ``bench.py --pipe-peaks``
+uses (a measurement tool, not part of the ES-step library).
 
-Each translation unit is compiled by nvcc in parallel, then linked into one
-shared library with the CUDA runtime linked statically, so the library has no
-dependency beyond the driver. ptxas register/spill reports go to
+Each translation unit is compiled by nvcc in parallel, then linked into its
+shared library with the CUDA runtime linked statically, so neither library has
+a dependency beyond the driver. ptxas register/spill reports go to
 ``_build/ptxas.log``.
 
     python -m paper_2608_17310_gb300.build [--force]
@@ -20,8 +22,10 @@ CSRC = os.path.join(PKG, "csrc")
 INCLUDE = os.path.join(ROOT, "include")
 BUILD = os.path.join(PKG, "_build")
 LIB = os.path.join(BUILD, "libesopt.so")
+PROBE_LIB = os.path.join(BUILD, "libesprobe.so")
 
 SOURCES = ["es_host.cu", "es_kernels.cu", "es_noalloc.cu"]
+PROBE_SOURCES = ["es_probes.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 NVCC_FLAGS = ["-std=c++17", "-O3", "-lineinfo", "-Xcompiler", "-fPIC,-O2",
               "-Xptxas", "-v", f"-I{INCLUDE}"]
@@ -42,9 +46,9 @@ def _deps():
 
 
 def up_to_date() -> bool:
-    if not os.path.exists(LIB):
+    if not (os.path.exists(LIB) and os.path.exists(PROBE_LIB)):
         return False
-    t = os.path.getmtime(LIB)
+    t = min(os.path.getmtime(LIB), os.path.getmtime(PROBE_LIB))
     return all(os.path.getmtime(f) <= t for f in _deps())
 
 
@@ -54,15 +58,15 @@ def build_library(force: bool = False, verbose: bool = False) -> str:
     os.makedirs(BUILD, exist_ok=True)
     cc = nvcc()
     procs = []
-    objs = []
-    for src in SOURCES:
+    objs = {}
+    for src in SOURCES + PROBE_SOURCES:
         obj = os.path.join(BUILD, os.path.splitext(src)[0] + ".o")
         cmd = [cc, *ARCH, *NVCC_FLAGS, "-c", os.path.join(CSRC, src), "-o", obj]
         if verbose:
             print(" ".join(cmd), flush=True)
         procs.append((src, subprocess.Popen(cmd, stdout=subprocess.PIPE,
                                             stderr=subprocess.STDOUT, text=True)))
-        objs.append(obj)
+        objs[src] = obj
     logs = []
     failed = []
     for src, p in procs:
@@ -74,12 +78,13 @@ def build_library(force: bool = False, verbose: bool = False) -> str:
         f.write("\n".join(logs))
     if failed:
         raise RuntimeError("nvcc failed for " + ", ".join(failed) + ":\n" + "\n".join(logs))
-    tmp = LIB + f".{os.getpid()}.tmp"
-    link = [cc, *ARCH, "-shared", "-o", tmp, *objs]
-    if verbose:
-        print(" ".join(link), flush=True)
-    subprocess.run(link, check=True)
-    os.replace(tmp, LIB)
+    for lib, srcs in ((LIB, SOURCES), (PROBE_LIB, PROBE_SOURCES)):
+        tmp = lib + f".{os.getpid()}.tmp"
+        link = [cc, *ARCH, "-shared", "-o", tmp, *(objs[s] for s in srcs)]
+        if verbose:
+            print(" ".join(link), flush=True)
+        subprocess.run(link, check=True)
+        os.replace(tmp, lib)
     return LIB
 
 

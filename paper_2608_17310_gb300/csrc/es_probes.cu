@@ -1,0 +1,413 @@
+// Register-only throughput probes of the SM pipes that bound the noise
+// generator (a measurement tool behind `bench.py --pipe-peaks`; not part of the
+// ES-step library and not linked into it).
+//
+// Every probe runs `iters` iterations of a fixed instruction pattern on
+// independent dependency chains held in registers: no memory traffic besides
+// one timing record per CTA. Each CTA times itself in SM clock cycles
+// (clock64) and in nanoseconds (globaltimer), so a rate comes out per SM per
+// clock, independent of the clock the GPU happened to run at.
+//
+// Probes:
+//   single pipes   mad.wide.u32 (the 32x32->64-bit product of each Philox
+//                  round), mad.hi.u32, mad.lo.u32, lop3 (the round's
+//                  three-input XOR), fma.rn.f32, packed fma.rn.f32x2, and MUFU
+//                  lg2/ex2 pairs (the transcendental unit Box-Muller uses);
+//   mixes          two pipes interleaved in one thread, in fixed ratios; the
+//                  ratio 9 products : 4 MUFU is the generator's (18 products
+//                  and 8 transcendentals per Philox block of 4 Gaussians), with
+//                  each product as one mad.wide.u32 or as a mad.hi.u32 +
+//                  mad.lo.u32 pair (the form the library uses);
+//   warp split     even warps run mad.wide chains and odd warps MUFU chains
+//                  (or only one half runs): whether the two pipes overlap at
+//                  all when their instructions come from different warps;
+//   generator      the library's own Philox4x32-10 (es_noise.cuh) in blocks,
+//                  and the full generator (Philox + Box-Muller) in Gaussians.
+#include <cuda_runtime.h>
+
+#include <cstdint>
+
+#include "es_noise.cuh"
+
+namespace {
+
+constexpr int kThreads = 256;
+constexpr uint32_t kMul = 0xD2511F53u;
+
+enum Probe : int {
+  kImadWide = 0,
+  kImadHi,
+  kImadLo,
+  kLop3,
+  kFfma,
+  kFfma2,
+  kMufu,
+  kMixImadMufu,
+  kMixImadFfma,
+  kMixImadLop3,
+  kMixMufuFfma,
+  kMixHiLo,
+  kMixHiLoMufu,
+  kSplitImad,
+  kSplitMufu,
+  kSplitBoth,
+  kPhilox,
+  kGenerator,
+  kProbeCount
+};
+
+// Name, unit of one op, ops per active thread per iteration, and the share of
+// threads that run (the split probes use half of the warps).
+struct ProbeInfo {
+  const char* name;
+  const char* unit;
+  double ops_per_iter;
+  double active;
+};
+
+// The MUFU half of a split probe runs iters / kSplitMufuDiv iterations, which
+// makes both halves take about as long when run alone.
+constexpr int kSplitMufuDiv = 4;
+
+const ProbeInfo kInfo[kProbeCount] = {
+    {"imad_wide", "mad.wide.u32", 8, 1},
+    {"imad_hi", "mad.hi.u32", 8, 1},
+    {"imad_lo", "mad.lo.u32", 8, 1},
+    {"lop3", "lop3.b32", 8, 1},
+    {"ffma", "fma.rn.f32", 8, 1},
+    {"ffma2", "fma.rn.f32x2 (2 lanes)", 8, 1},
+    {"mufu", "MUFU lg2 or ex2", 16, 1},
+    {"mix_imad_wide_mufu_9_4", "mad.wide.u32 (with 4 MUFU per 9)", 9, 1},
+    {"mix_imad_wide_ffma_1_2", "mad.wide.u32 (with 2 fma.rn.f32 each)", 8, 1},
+    {"mix_imad_wide_lop3_1_1", "mad.wide.u32 (with 1 lop3.b32 each)", 8, 1},
+    {"mix_mufu_ffma_1_4", "MUFU (with 4 fma.rn.f32 each)", 8, 1},
+    {"mix_imad_hi_lo_1_1", "mad.hi.u32 + mad.lo.u32 pair", 8, 1},
+    {"mix_imad_hi_lo_mufu_9_4", "mad.hi.u32 + mad.lo.u32 pair (with 4 MUFU per 9)", 9, 1},
+    {"split_imad_wide_only", "mad.wide.u32 (even warps; odd warps idle)", 8, 0.5},
+    {"split_mufu_only", "MUFU (odd warps; even warps idle)", 16.0 / kSplitMufuDiv, 0.5},
+    {"split_both", "warp-iterations (even warps mad.wide, odd warps MUFU)", 1, 1},
+    {"philox", "Philox4x32-10 block", 2, 1},
+    {"generator", "Gaussian (Philox4x32-10 + Box-Muller)", 8, 1},
+};
+
+__device__ __forceinline__ uint64_t mad_wide(uint32_t a, uint64_t c) {
+  uint64_t d;
+  asm volatile("mad.wide.u32 %0, %1, %2, %3;" : "=l"(d) : "r"(a), "r"(kMul), "l"(c));
+  return d;
+}
+__device__ __forceinline__ uint32_t mad_hi(uint32_t a, uint32_t c) {
+  uint32_t d;
+  asm volatile("mad.hi.u32 %0, %1, %2, %3;" : "=r"(d) : "r"(a), "r"(kMul), "r"(c));
+  return d;
+}
+__device__ __forceinline__ uint32_t mad_lo(uint32_t a, uint32_t c) {
+  uint32_t d;
+  asm volatile("mad.lo.u32 %0, %1, %2, %3;" : "=r"(d) : "r"(a), "r"(kMul), "r"(c));
+  return d;
+}
+__device__ __forceinline__ uint32_t xor3(uint32_t a, uint32_t b, uint32_t c) {
+  uint32_t d;
+  asm volatile("lop3.b32 %0, %1, %2, %3, 0x96;" : "=r"(d) : "r"(a), "r"(b), "r"(c));
+  return d;
+}
+__device__ __forceinline__ float ffma(float a, float b, float c) {
+  float d;
+  asm volatile("fma.rn.f32 %0, %1, %2, %3;" : "=f"(d) : "f"(a), "f"(b), "f"(c));
+  return d;
+}
+// ex2(lg2(a)): two MUFU operations that return (about) a, so the chain stays
+// finite and positive for any number of iterations.
+__device__ __forceinline__ float mufu2(float a) {
+  float l, e;
+  asm volatile("lg2.approx.ftz.f32 %0, %1;" : "=f"(l) : "f"(a));
+  asm volatile("ex2.approx.ftz.f32 %0, %1;" : "=f"(e) : "f"(l));
+  return e;
+}
+
+template <int P>
+__global__ void __launch_bounds__(kThreads)
+probe_kernel(int iters, uint32_t seed, unsigned long long* __restrict__ rec,
+             uint32_t* __restrict__ sink) {
+  const uint32_t t = seed + threadIdx.x * 0x9E3779B9u + blockIdx.x;
+  uint64_t w[9];
+  uint32_t x[8], y[8];
+  float f[8], m[4];
+  float2 f2[8];
+#pragma unroll
+  for (int k = 0; k < 9; ++k) w[k] = t * (2u * k + 1u);
+#pragma unroll
+  for (int k = 0; k < 8; ++k) {
+    x[k] = t + 977u * k;
+    y[k] = t ^ (0x85EBCA6Bu * k);
+    f[k] = 1.0f + (t & 0xFFu) * 1e-4f + k * 1e-3f;
+    f2[k] = make_float2(f[k], f[k] + 0.5f);
+  }
+#pragma unroll
+  for (int k = 0; k < 4; ++k) m[k] = 1.5f + (t & 0xFFu) * 1e-3f + k * 0.25f;
+  const float fb = 0.999f + (seed & 1) * 1e-7f, fc = 1e-3f * (seed & 3);
+  const int warp = threadIdx.x >> 5;
+
+  __syncthreads();
+  unsigned long long c0 = 0, n0 = 0;
+  if (threadIdx.x == 0) {
+    c0 = clock64();
+    asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(n0));
+  }
+
+  if constexpr (P == kImadWide || P == kSplitImad) {
+    if (P == kImadWide || (warp & 1) == 0) {
+#pragma unroll 1
+      for (int i = 0; i < iters; ++i)
+#pragma unroll
+        for (int k = 0; k < 8; ++k) w[k] = mad_wide(static_cast<uint32_t>(w[k]), w[k]);
+    }
+  } else if constexpr (P == kImadHi) {
+#pragma unroll 1
+    for (int i = 0; i < iters; ++i)
+#pragma unroll
+      for (int k = 0; k < 8; ++k) x[k] = mad_hi(x[k], y[k]);
+  } else if constexpr (P == kImadLo) {
+#pragma unroll 1
+    for (int i = 0; i < iters; ++i)
+#pragma unroll
+      for (int k = 0; k < 8; ++k) x[k] = mad_lo(x[k], y[k]);
+  } else if constexpr (P == kLop3) {
+#pragma unroll 1
+    for (int i = 0; i < iters; ++i)
+#pragma unroll
+      for (int k = 0; k < 8; ++k) x[k] = xor3(x[k], y[k], x[(k + 1) & 7]);
+  } else if constexpr (P == kFfma) {
+#pragma unroll 1
+    for (int i = 0; i < iters; ++i)
+#pragma unroll
+      for (int k = 0; k < 8; ++k) f[k] = ffma(f[k], fb, fc);
+  } else if constexpr (P == kFfma2) {
+    const float2 b2 = make_float2(fb, fb), c2 = make_float2(fc, fc);
+#pragma unroll 1
+    for (int i = 0; i < iters; ++i)
+#pragma unroll
+      for (int k = 0; k < 8; ++k) f2[k] = __ffma2_rn(f2[k], b2, c2);
+  } else if constexpr (P == kMufu || P == kSplitMufu) {
+    if (P == kMufu || (warp & 1) == 1) {
+      const int n = P == kMufu ? iters : iters / kSplitMufuDiv;
+#pragma unroll 1
+      for (int i = 0; i < n; ++i)
+#pragma unroll
+        for (int k = 0; k < 8; ++k) f[k] = mufu2(f[k]);
+    }
+  } else if constexpr (P == kSplitBoth) {
+    if ((warp & 1) == 0) {
+#pragma unroll 1
+      for (int i = 0; i < iters; ++i)
+#pragma unroll
+        for (int k = 0; k < 8; ++k) w[k] = mad_wide(static_cast<uint32_t>(w[k]), w[k]);
+    } else {
+#pragma unroll 1
+      for (int i = 0; i < iters / kSplitMufuDiv; ++i)
+#pragma unroll
+        for (int k = 0; k < 8; ++k) f[k] = mufu2(f[k]);
+    }
+  } else if constexpr (P == kMixImadMufu) {
+#pragma unroll 1
+    for (int i = 0; i < iters; ++i) {
+#pragma unroll
+      for (int k = 0; k < 9; ++k) w[k] = mad_wide(static_cast<uint32_t>(w[k]), w[k]);
+      m[0] = mufu2(m[0]);
+      m[1] = mufu2(m[1]);
+    }
+  } else if constexpr (P == kMixImadFfma) {
+#pragma unroll 1
+    for (int i = 0; i < iters; ++i) {
+#pragma unroll
+      for (int k = 0; k < 8; ++k) {
+        w[k] = mad_wide(static_cast<uint32_t>(w[k]), w[k]);
+        f[k] = ffma(ffma(f[k], fb, fc), fb, fc);
+      }
+    }
+  } else if constexpr (P == kMixImadLop3) {
+#pragma unroll 1
+    for (int i = 0; i < iters; ++i) {
+#pragma unroll
+      for (int k = 0; k < 8; ++k) {
+        w[k] = mad_wide(static_cast<uint32_t>(w[k]), w[k]);
+        x[k] = xor3(x[k], y[k], x[(k + 1) & 7]);
+      }
+    }
+  } else if constexpr (P == kMixMufuFfma) {
+#pragma unroll 1
+    for (int i = 0; i < iters; ++i) {
+#pragma unroll
+      for (int k = 0; k < 4; ++k) m[k] = mufu2(m[k]);
+#pragma unroll
+      for (int k = 0; k < 8; ++k) f[k] = ffma(ffma(ffma(ffma(f[k], fb, fc), fb, fc), fb, fc), fb, fc);
+    }
+  } else if constexpr (P == kMixHiLo) {
+#pragma unroll 1
+    for (int i = 0; i < iters; ++i) {
+#pragma unroll
+      for (int k = 0; k < 8; ++k) {
+        x[k] = mad_hi(x[k], y[(k + 3) & 7]);
+        y[k] = mad_lo(y[k], x[(k + 5) & 7]);
+      }
+    }
+  } else if constexpr (P == kMixHiLoMufu) {
+#pragma unroll 1
+    for (int i = 0; i < iters; ++i) {
+#pragma unroll
+      for (int k = 0; k < 8; ++k) {
+        x[k] = mad_hi(x[k], y[(k + 3) & 7]);
+        y[k] = mad_lo(y[k], x[(k + 5) & 7]);
+      }
+      w[8] = (static_cast<uint64_t>(mad_hi(static_cast<uint32_t>(w[8]), x[0])) << 32) |
+             mad_lo(static_cast<uint32_t>(w[8] >> 32), y[0]);
+      m[0] = mufu2(m[0]);
+      m[1] = mufu2(m[1]);
+    }
+  } else if constexpr (P == kPhilox) {
+    const esopt::PhiloxTile pt = esopt::philox_tile(0u, esopt::philox_key(seed));
+    uint32_t j = t * 2u;
+#pragma unroll 1
+    for (int i = 0; i < iters; ++i) {
+      const uint4 a = esopt::philox_block_tile(j, pt);
+      const uint4 b = esopt::philox_block_tile(j + 1u, pt);
+      x[0] ^= a.x ^ b.x;
+      x[1] ^= a.y ^ b.y;
+      x[2] ^= a.z ^ b.z;
+      x[3] ^= a.w ^ b.w;
+      j += 0x20000u;
+    }
+  } else if constexpr (P == kGenerator) {
+    const esopt::PhiloxTile pt = esopt::philox_tile(0u, esopt::philox_key(seed));
+    uint32_t j = t * 2u;
+    float2 s0 = make_float2(0.f, 0.f), s1 = s0;
+#pragma unroll 1
+    for (int i = 0; i < iters; ++i) {
+#pragma unroll
+      for (int b = 0; b < 2; ++b) {
+        const esopt::Polar2 p = esopt::polar2(esopt::philox_block_tile(j + b, pt));
+        s0 = __ffma2_rn(make_float2(p.r.x, p.r.x), make_float2(p.c.x, p.s.x), s0);
+        s1 = __ffma2_rn(make_float2(p.r.y, p.r.y), make_float2(p.c.y, p.s.y), s1);
+      }
+      j += 0x20000u;
+    }
+    f[0] = s0.x + s0.y + s1.x + s1.y;
+  }
+
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    unsigned long long n1;
+    const unsigned long long c1 = clock64();
+    asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(n1));
+    rec[2 * blockIdx.x] = c1 - c0;
+    rec[2 * blockIdx.x + 1] = n1 - n0;
+  }
+  // Fold every chain into one word so that no chain is dead code; the store
+  // happens only for a value that depends on all of them and the seed.
+  uint32_t s = 0;
+#pragma unroll
+  for (int k = 0; k < 9; ++k) s ^= static_cast<uint32_t>(w[k] ^ (w[k] >> 32));
+#pragma unroll
+  for (int k = 0; k < 8; ++k)
+    s ^= x[k] ^ __float_as_uint(f[k]) ^ __float_as_uint(f2[k].x) ^ __float_as_uint(f2[k].y);
+#pragma unroll
+  for (int k = 0; k < 4; ++k) s ^= __float_as_uint(m[k]);
+  if (s == seed * 0x2545F491u + 0x1234567u) sink[0] = s;
+}
+
+template <int P>
+void* kernel_of() {
+  return reinterpret_cast<void*>(probe_kernel<P>);
+}
+
+void* const kKernels[kProbeCount] = {
+    kernel_of<0>(),  kernel_of<1>(),  kernel_of<2>(),  kernel_of<3>(),
+    kernel_of<4>(),  kernel_of<5>(),  kernel_of<6>(),  kernel_of<7>(),
+    kernel_of<8>(),  kernel_of<9>(),  kernel_of<10>(), kernel_of<11>(),
+    kernel_of<12>(), kernel_of<13>(), kernel_of<14>(), kernel_of<15>(),
+    kernel_of<16>(), kernel_of<17>(),
+};
+
+}  // namespace
+
+extern "C" {
+
+int esprobe_count(void) { return kProbeCount; }
+
+const char* esprobe_name(int probe) {
+  return probe >= 0 && probe < kProbeCount ? kInfo[probe].name : "";
+}
+
+const char* esprobe_unit(int probe) {
+  return probe >= 0 && probe < kProbeCount ? kInfo[probe].unit : "";
+}
+
+// Runs probe `probe` on the current device with ctas_per_sm CTAs of 256
+// threads on every SM (all resident at once; fewer if the probe's registers
+// allow fewer) for `iters` iterations, after one untimed launch.
+// out[0..6] = milliseconds (CUDA events), mean SM cycles per CTA, SM clock in
+// MHz (cycles / globaltimer ns), ops per clock per SM, ops in total, active
+// threads per SM, CTAs per SM used. Returns 0, -1 for a bad argument, else the
+// cudaError_t.
+int esprobe_run(int probe, int ctas_per_sm, int iters, double* out) {
+  if (probe < 0 || probe >= kProbeCount || ctas_per_sm < 1 || iters < 1 || out == nullptr)
+    return -1;
+  int dev = 0, sms = 0, fit = 0;
+  cudaError_t err = cudaGetDevice(&dev);
+  if (err == cudaSuccess) err = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  if (err == cudaSuccess)
+    err = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&fit, kKernels[probe], kThreads, 0);
+  if (err != cudaSuccess) return static_cast<int>(err);
+  if (fit < 1) return -1;
+  if (fit < ctas_per_sm) ctas_per_sm = fit;
+  const int grid = sms * ctas_per_sm;
+  unsigned long long* rec = nullptr;
+  uint32_t* sink = nullptr;
+  cudaEvent_t e0 = nullptr, e1 = nullptr;
+  err = cudaMalloc(&rec, sizeof(unsigned long long) * 2 * grid);
+  if (err == cudaSuccess) err = cudaMalloc(&sink, sizeof(uint32_t));
+  if (err == cudaSuccess) err = cudaEventCreate(&e0);
+  if (err == cudaSuccess) err = cudaEventCreate(&e1);
+  unsigned long long* host = new unsigned long long[2 * grid];
+  float ms = 0.0f;
+  if (err == cudaSuccess) {
+    uint32_t seed = 0x51ED270Bu;
+    int warm_iters = iters / 8 > 0 ? iters / 8 : 1;
+    void* warm[] = {&warm_iters, &seed, &rec, &sink};
+    err = cudaLaunchKernel(kKernels[probe], dim3(grid), dim3(kThreads), warm, 0, 0);
+    if (err == cudaSuccess) err = cudaEventRecord(e0, 0);
+    void* args[] = {&iters, &seed, &rec, &sink};
+    if (err == cudaSuccess)
+      err = cudaLaunchKernel(kKernels[probe], dim3(grid), dim3(kThreads), args, 0, 0);
+    if (err == cudaSuccess) err = cudaEventRecord(e1, 0);
+    if (err == cudaSuccess) err = cudaEventSynchronize(e1);
+    if (err == cudaSuccess) err = cudaEventElapsedTime(&ms, e0, e1);
+    if (err == cudaSuccess)
+      err = cudaMemcpy(host, rec, sizeof(unsigned long long) * 2 * grid, cudaMemcpyDeviceToHost);
+  }
+  if (err == cudaSuccess) {
+    double cyc = 0.0, ns = 0.0;
+    for (int b = 0; b < grid; ++b) {
+      cyc += static_cast<double>(host[2 * b]);
+      ns += static_cast<double>(host[2 * b + 1]);
+    }
+    cyc /= grid;
+    ns /= grid;
+    const double threads_per_sm = static_cast<double>(ctas_per_sm) * kThreads;
+    const double ops = kInfo[probe].ops_per_iter * iters * threads_per_sm * kInfo[probe].active;
+    out[0] = ms;
+    out[1] = cyc;
+    out[2] = ns > 0.0 ? cyc / ns * 1e3 : 0.0;
+    out[3] = ops / cyc;
+    out[4] = ops * sms;
+    out[5] = threads_per_sm * kInfo[probe].active;
+    out[6] = ctas_per_sm;
+  }
+  delete[] host;
+  if (e0) cudaEventDestroy(e0);
+  if (e1) cudaEventDestroy(e1);
+  cudaFree(rec);
+  cudaFree(sink);
+  return static_cast<int>(err);
+}
+
+}  // extern "C"
