@@ -8,6 +8,7 @@ synthetic parameter set shaped like the paper's workloads.
     python bench.py --replay [--population N] [--generations K]
     python bench.py --antithetic
     python bench.py --generator [--gen-log2 31]
+    python bench.py --pipe-peaks
 
 Prints one JSON line (rank 0). `value` is measured with the inputs resident in
 HBM; `e2e` is the same metric with the parameters in pinned host memory and
@@ -49,12 +50,14 @@ def parse():
     p.add_argument("--gpus", type=int, default=1)
     p.add_argument("--steps", type=int, default=5)
     p.add_argument("--warmup", type=int, default=3)
-    p.add_argument("--workload", default="qwen27b", choices=["qwen27b", "qwen4b", "qwen4b_f32", "qwen4b_4layer", "toy"])
+    p.add_argument("--workload", default="qwen27b",
+                   choices=["qwen27b", "qwen4b", "qwen4b_f32", "qwen4b_fp8", "qwen4b_4layer", "toy"])
     p.add_argument("--population", type=int, default=None, help="override N")
     p.add_argument("--impl", default="ours", choices=["ours", "reference"])
     p.add_argument("--no-e2e", action="store_true")
     p.add_argument("--no-cpu-baseline", action="store_true")
-    p.add_argument("--e2e-steps", type=int, default=2)
+    p.add_argument("--e2e-steps", type=int, default=None,
+                   help="generations timed by the e2e leg (default: --steps, at least 5)")
     p.add_argument("--unfused", action="store_true",
                    help="separate es_restore / es_perturb launches instead of es_restore_perturb")
     p.add_argument("--sweep", action="store_true",
@@ -71,10 +74,16 @@ def parse():
                         "(2^31 Gaussians per launch) and es_noise_bits")
     p.add_argument("--gen-log2", type=int, default=31,
                    help="--generator: 2^k Gaussians per es_noise_fill launch")
+    p.add_argument("--pipe-peaks", action="store_true",
+                   help="instead of the step: the register-only pipe probes (integer "
+                        "multiply, MUFU, FMA, LOP3, their mixes, a warp-split overlap test, "
+                        "the generator) in ops per clock per SM")
     p.add_argument("--antithetic", action="store_true",
                    help="instead of the step: a generation of N/2 antithetic pairs (the +/- "
                         "flip as one es_restore_perturb on one seed)")
     args = p.parse_args()
+    if args.e2e_steps is None:
+        args.e2e_steps = max(5, args.steps)
     if (args.sweep or args.replay) and "--workload" not in " ".join(sys.argv):
         args.workload = "qwen4b"
     return args
@@ -187,12 +196,29 @@ class ClockSampler:
 L2_BYTES = 129 * 1024 * 1024     # GB300 L2
 
 
+ELEM_BYTES = {"bf16": 2, "f32": 4, "e4m3": 1}
+
+
+def param_set(es, workload: str):
+    """(flat buffer, views, plan, bytes per element) of a workload's parameter
+    set on the current CUDA device; FP8 sets get a scaled plan."""
+    import torch
+    wl = I.WORKLOADS[workload]
+    specs = I.shapes_for(workload)
+    if wl.dtype == "e4m3":
+        flat, params, scales = I.init_params_flat_e4m3(specs, "cuda", seed=0)
+        return flat, params, es.plan_from_tensors(params, scales=scales), 1
+    dtype = torch.bfloat16 if wl.dtype == "bf16" else torch.float32
+    flat, params = I.init_params_flat(specs, dtype, "cuda", seed=0)
+    return flat, params, es.plan_from_tensors(params), ELEM_BYTES[wl.dtype]
+
+
 def workload_config(workload: str, n: int, world: int) -> dict:
     """The `config` object of the JSON line (shared by both arms)."""
     wl = I.WORKLOADS[workload]
     specs = I.shapes_for(workload)
     P = sum(s.numel for s in specs)
-    esize = 2 if wl.dtype == "bf16" else 4
+    esize = ELEM_BYTES[wl.dtype]
     return {"workload": workload, "params": P, "population": n, "storage": wl.dtype,
             "segments": len(specs), "description": wl.description, "alpha": wl.alpha,
             "l2": ("inputs larger than L2 (%.1f GB of parameters)" % (P * esize / 1e9)
@@ -308,13 +334,14 @@ def gauss_per_elem(kind, n):
     return n + 1 if kind == "update_perturb" else n
 # Philox4x32-10 on counter (j_lo, j_hi, 0, 0): 10 rounds x 2 products of
 # 32x32->64 bits per 4 outputs, less the first round's product by 0 and the
-# second round's product of (key, j_hi) alone (shared by a tile): 18 products,
-# each two 32-bit multiplies (high and low word), i.e. 9 per Gaussian.
+# second round's product of (key, j_hi) alone (shared by a tile): 18 products
+# (mad.wide.u32), each two 32-bit multiplies (high and low word), i.e. 9 per
+# Gaussian. The nominal rate is 64 32-bit multiplies per clock per SM.
 IMUL_PER_GAUSS = 9
+WIDE_PER_GAUSS = IMUL_PER_GAUSS / 2
 IMUL_PER_CLK_SM = 64
-# Box-Muller: log2, sqrt, sin and cos per pair on the MUFU pipe (16 per clock
-# per SM): 2 per Gaussian. On sm_103a the integer-multiply and MUFU work of one
-# SM sub-partition does not overlap (measured), so their times add.
+# Box-Muller: log2, sqrt, sin and cos per pair on the MUFU pipe (nominal 16
+# per clock per SM): 2 per Gaussian.
 MUFU_PER_GAUSS = 2
 MUFU_PER_CLK_SM = 16
 
@@ -403,11 +430,7 @@ def run_ours(args, rank, world, dist):
     torch.cuda.init()
     wl = I.WORKLOADS[args.workload]
     n = args.population or wl.population
-    specs = I.shapes_for(args.workload)
-    dtype = torch.bfloat16 if wl.dtype == "bf16" else torch.float32
-    esize = 2 if wl.dtype == "bf16" else 4
-    flat, params = I.init_params_flat(specs, dtype, "cuda", seed=0)
-    plan = es.plan_from_tensors(params)
+    flat, params, plan, esize = param_set(es, args.workload)
     P = plan.numel
     stream = torch.cuda.current_stream()
     s_handle = stream.cuda_stream
@@ -443,7 +466,8 @@ def run_ours(args, rank, world, dist):
     per_step_ms = ms_max / args.steps
     value = world * P * n * args.steps / (ms_max / 1e3)
 
-    imul_peak, gauss_peak, shared_peak, sms, sm_max_mhz, hbm_gbs, peak_src = alu_peaks(torch, dev_index)
+    imul_peak, gauss_peak, shared_peak, sms, sm_max_mhz, hbm_gbs, peak_src, ceilings = \
+        alu_peaks(torch, dev_index)
     bytes_per_launch = 2 * esize * P
     kernels = {}
     for name in timers.names():
@@ -473,9 +497,10 @@ def run_ours(args, rank, world, dist):
                                f"{sm_max_mhz:.0f} MHz; {IMUL_PER_GAUSS} multiplies per Gaussian"}
     roof["imul_mufu_bound"] = {
         "gauss_per_s": shared_peak, "frac": d["gauss_per_s"] / shared_peak,
-        "source": f"integer-multiply and MUFU work issue from the same SM sub-partition "
-                  f"without overlap: {IMUL_PER_GAUSS}/{IMUL_PER_CLK_SM} + "
-                  f"{MUFU_PER_GAUSS}/{MUFU_PER_CLK_SM} SM-clocks per Gaussian"}
+        "source": "measured in this run: register-only probe of mad.wide.u32 and MUFU in the "
+                  "generator's ratio (9:4) in one thread, 4 CTAs per SM, scaled to the "
+                  "maximum SM clock (bench.py --pipe-peaks has every probe)"}
+    roof["measured_ceilings"] = ceilings
     roof["pipe_occupancy"] = pipe_occupancy(dom)
     roof.update({"kernel": d["kernel"], "hbm_frac": d["hbm_frac"], "alu_frac": d["alu_frac"],
                  "algorithmic_bytes_per_launch": bytes_per_launch,
@@ -510,15 +535,152 @@ def run_ours(args, rank, world, dist):
         print(json.dumps(out), flush=True)
 
 
-def alu_peaks(torch, dev_index):
-    """(imul32/s, Gaussians/s at the integer-multiply roofline, Gaussians/s at
-    the IMUL+MUFU bound, SM count, max SM MHz, HBM GB/s, peak source)."""
+def probe_lib():
+    """The register-only pipe probes (csrc/es_probes.cu, _build/libesprobe.so)."""
+    import ctypes
+    from paper_2608_17310_gb300 import build
+    build.build_library()
+    L = ctypes.CDLL(build.PROBE_LIB)
+    L.esprobe_count.restype = ctypes.c_int
+    L.esprobe_name.argtypes = [ctypes.c_int]
+    L.esprobe_name.restype = ctypes.c_char_p
+    L.esprobe_unit.argtypes = [ctypes.c_int]
+    L.esprobe_unit.restype = ctypes.c_char_p
+    L.esprobe_run.argtypes = [ctypes.c_int, ctypes.c_int, ctypes.c_int,
+                              ctypes.POINTER(ctypes.c_double)]
+    L.esprobe_run.restype = ctypes.c_int
+    return L
+
+
+def run_probe(L, name, ctas_per_sm=4, target_ms=20.0):
+    """One probe, its iteration count scaled so the timed launch takes about
+    target_ms. Rates are per SM per clock (the probe times itself in SM cycles)."""
+    import ctypes
+    ids = {L.esprobe_name(i).decode(): i for i in range(L.esprobe_count())}
+    pid = ids[name]
+    out = (ctypes.c_double * 7)()
+    iters = 256
+    for _ in range(2):
+        rc = L.esprobe_run(pid, ctas_per_sm, iters, out)
+        if rc != 0:
+            raise RuntimeError(f"probe {name}: esprobe_run returned {rc}")
+        if out[0] >= 0.5 * target_ms:
+            break
+        iters = max(256, int(iters * target_ms / max(out[0], 1e-3)) // 4 * 4)
+    return {"probe": name, "unit": L.esprobe_unit(pid).decode(), "ctas_per_sm": int(out[6]),
+            "iters": iters, "ms": out[0], "cycles": out[1], "sm_mhz": out[2],
+            "ops_per_clk_sm": out[3], "ops": out[4], "threads_per_sm": out[5]}
+
+
+def measured_ceilings(res, sms, sm_max_mhz):
+    """ALU ceilings of the generator from probe results (`res`: name -> run_probe
+    dict), in Gaussians/s at the maximum SM clock:
+      imad_wide      the integer-multiply pipe alone: mad.wide.u32 rate / 4.5;
+      mufu           the MUFU pipe alone: its rate / 2;
+      imad_mufu_mix  both in the generator's ratio (9 mad.wide : 4 MUFU) in one
+                     thread: the shared ceiling of this formulation;
+      generator      the library's full generator (Philox + Box-Muller) in
+                     registers, no memory traffic."""
+    hz = sms * sm_max_mhz * 1e6
+    out = {}
+    if "imad_wide" in res:
+        r = res["imad_wide"]["ops_per_clk_sm"]
+        out["imad_wide"] = {"ops_per_clk_sm": r, "imul32_per_clk_sm": 2 * r,
+                            "gauss_per_s": r / WIDE_PER_GAUSS * hz}
+    if "mufu" in res:
+        r = res["mufu"]["ops_per_clk_sm"]
+        out["mufu"] = {"ops_per_clk_sm": r, "gauss_per_s": r / MUFU_PER_GAUSS * hz}
+    if "mix_imad_wide_mufu_9_4" in res:
+        r = res["mix_imad_wide_mufu_9_4"]["ops_per_clk_sm"]
+        out["imad_mufu_mix"] = {"wide_per_clk_sm": r, "gauss_per_s": r / WIDE_PER_GAUSS * hz}
+        if "imad_wide" in out and "mufu" in out:
+            a, m = out["imad_wide"]["ops_per_clk_sm"], out["mufu"]["ops_per_clk_sm"]
+            additive = 1.0 / (WIDE_PER_GAUSS / a + MUFU_PER_GAUSS / m)
+            overlapped = min(a / WIDE_PER_GAUSS, m / MUFU_PER_GAUSS)
+            out["imad_mufu_mix"].update({
+                "gauss_per_s_if_additive": additive * hz,
+                "gauss_per_s_if_overlapped": overlapped * hz})
+    if "mix_imad_hi_lo_1_1" in res:
+        r = res["mix_imad_hi_lo_1_1"]["ops_per_clk_sm"]
+        out["imad_hi_lo"] = {"pairs_per_clk_sm": r, "imul32_per_clk_sm": 2 * r,
+                             "gauss_per_s": r / WIDE_PER_GAUSS * hz}
+    if "mix_imad_hi_lo_mufu_9_4" in res:
+        r = res["mix_imad_hi_lo_mufu_9_4"]["ops_per_clk_sm"]
+        out["imad_hi_lo_mufu_mix"] = {"pairs_per_clk_sm": r, "gauss_per_s": r / WIDE_PER_GAUSS * hz}
+    if "generator" in res:
+        r = res["generator"]["ops_per_clk_sm"]
+        out["generator"] = {"gauss_per_clk_sm": r, "gauss_per_s": r * hz}
+    if all(k in res for k in ("split_imad_wide_only", "split_mufu_only", "split_both")):
+        ti = res["split_imad_wide_only"]["cycles"]
+        tm = res["split_mufu_only"]["cycles"]
+        tb = res["split_both"]["cycles"]
+        out["warp_split"] = {"cycles_imad_only": ti, "cycles_mufu_only": tm, "cycles_both": tb,
+                             "overlap": (ti + tm - tb) / min(ti, tm)}
+    return out
+
+
+CEILING_PROBES = ("imad_wide", "mufu", "mix_imad_wide_mufu_9_4", "mix_imad_hi_lo_1_1",
+                  "mix_imad_hi_lo_mufu_9_4", "generator")
+
+
+def alu_peaks(torch, dev_index, probes=True):
+    """(imul32/s at the nominal integer-multiply rate, Gaussians/s at that
+    roofline, Gaussians/s at the measured shared IMUL+MUFU ceiling, SM count,
+    max SM MHz, HBM GB/s, peak source, measured ceilings).
+
+    The roofline is the nominal one: 64 32-bit multiplies per clock per SM x
+    SMs x the maximum SM clock, 9 multiplies per Gaussian. The shared ceiling is
+    measured live by the register-only probes (the generator's mix of
+    mad.wide.u32 and MUFU in one thread); without probes it is None."""
     hbm_gbs, sm_max_mhz, peak_src = peaks()
     sms = torch.cuda.get_device_properties(dev_index).multi_processor_count
     imul_peak = sms * IMUL_PER_CLK_SM * sm_max_mhz * 1e6
-    shared_peak = sms * sm_max_mhz * 1e6 / (IMUL_PER_GAUSS / IMUL_PER_CLK_SM +
-                                             MUFU_PER_GAUSS / MUFU_PER_CLK_SM)
-    return imul_peak, imul_peak / IMUL_PER_GAUSS, shared_peak, sms, sm_max_mhz, hbm_gbs, peak_src
+    ceilings = {}
+    shared_peak = None
+    if probes:
+        L = probe_lib()
+        res = {name: run_probe(L, name, 4, 10.0) for name in CEILING_PROBES}
+        ceilings = measured_ceilings(res, sms, sm_max_mhz)
+        ceilings["source"] = ("bench.py probes (csrc/es_probes.cu): register-only loops, 4 CTAs "
+                              "of 256 threads per SM, rates in SM cycles scaled to the maximum "
+                              "SM clock")
+        shared_peak = ceilings["imad_mufu_mix"]["gauss_per_s"]
+    return (imul_peak, imul_peak / IMUL_PER_GAUSS, shared_peak, sms, sm_max_mhz, hbm_gbs,
+            peak_src, ceilings)
+
+
+def run_pipe_peaks(args, rank, world, dist):
+    """Every register-only probe of csrc/es_probes.cu: single pipes, two-pipe
+    mixes, the warp-split overlap test and the library's generator, at 4 CTAs of
+    256 threads per SM, and at 1, 2 and 8 (where the registers allow) for the
+    main ones. Rates are per SM per clock;
+    ceilings are scaled to the maximum SM clock."""
+    import torch
+    torch.cuda.init()
+    dev_index = torch.cuda.current_device()
+    hbm_gbs, sm_max_mhz, peak_src = peaks()
+    sms = torch.cuda.get_device_properties(dev_index).multi_processor_count
+    L = probe_lib()
+    names = [L.esprobe_name(i).decode() for i in range(L.esprobe_count())]
+    res, occupancy = {}, []
+    with ClockSampler(dev_index) as clk:
+        for name in names:
+            res[name] = run_probe(L, name, 4, 25.0)
+        for name in ("imad_wide", "mufu", "mix_imad_wide_mufu_9_4", "mix_imad_hi_lo_1_1",
+                     "mix_imad_hi_lo_mufu_9_4", "philox", "generator"):
+            for ctas in (1, 2, 8):
+                occupancy.append(run_probe(L, name, ctas, 25.0))
+    out = {"mode": "pipe_peaks", "metric": "ops per clock per SM of register-only pipe probes",
+           "unit": "ops/clk/SM", "n_gpus": 1, "data": "synthetic (register-only loops)",
+           "config": {"threads_per_cta": 256, "ctas_per_sm": 4, "sms": sms,
+                      "sm_max_mhz": sm_max_mhz,
+                      "nominal": {"imul32_per_clk_sm": IMUL_PER_CLK_SM,
+                                  "mufu_per_clk_sm": MUFU_PER_CLK_SM}},
+           "probes": [res[n] for n in names], "occupancy": occupancy,
+           "ceilings": measured_ceilings(res, sms, sm_max_mhz),
+           "gpu_launches": 2 * (len(res) + len(occupancy)) * 2, "clocks": clk.summary()}
+    if rank == 0:
+        print(json.dumps(out), flush=True)
 
 
 def run_sweep(args, rank, world, dist):
@@ -533,15 +695,12 @@ def run_sweep(args, rank, world, dist):
     dev_index = torch.cuda.current_device()
     torch.cuda.init()
     wl = I.WORKLOADS[args.workload]
-    specs = I.shapes_for(args.workload)
-    dtype = torch.bfloat16 if wl.dtype == "bf16" else torch.float32
-    esize = 2 if wl.dtype == "bf16" else 4
-    flat, params = I.init_params_flat(specs, dtype, "cuda", seed=0)
-    plan = es.plan_from_tensors(params)
+    flat, params, plan, esize = param_set(es, args.workload)
     P = plan.numel
     stream = torch.cuda.current_stream()
     s_handle = stream.cuda_stream
-    imul_peak, gauss_peak, shared_peak, sms, sm_max_mhz, hbm_gbs, peak_src = alu_peaks(torch, dev_index)
+    imul_peak, gauss_peak, shared_peak, sms, sm_max_mhz, hbm_gbs, peak_src, _ = \
+        alu_peaks(torch, dev_index)
     bytes_per_launch = 2 * esize * P
     pops = [int(x) for x in args.populations.split(",") if x.strip()]
     points = []
@@ -610,7 +769,7 @@ def _timed(torch, stream, fn, reps):
 
 
 def _rates(P, gaussians_per_param, bytes_total, ms, peaks_):
-    imul_peak, gauss_peak, shared_peak, _, _, hbm_gbs, _ = peaks_
+    imul_peak, gauss_peak, shared_peak, _, _, hbm_gbs, _, _ = peaks_
     gps = gaussians_per_param * P / (ms / 1e3)
     gbs = bytes_total / (ms / 1e3) / 1e9
     return {"ms": ms, "gauss_per_s": gps, "gbs": gbs, "hbm_frac": gbs / hbm_gbs,
@@ -629,11 +788,7 @@ def run_replay(args, rank, world, dist):
     wl = I.WORKLOADS[args.workload]
     n = args.population or wl.population
     K = args.generations
-    specs = I.shapes_for(args.workload)
-    dtype = torch.bfloat16 if wl.dtype == "bf16" else torch.float32
-    esize = 2 if wl.dtype == "bf16" else 4
-    flat, params = I.init_params_flat(specs, dtype, "cuda", seed=0)
-    plan = es.plan_from_tensors(params)
+    flat, params, plan, esize = param_set(es, args.workload)
     P = plan.numel
     stream = torch.cuda.current_stream()
     sh = stream.cuda_stream
@@ -760,11 +915,7 @@ def run_antithetic(args, rank, world, dist):
     torch.cuda.init()
     wl = I.WORKLOADS[args.workload]
     pairs = (args.population or wl.population) // 2
-    specs = I.shapes_for(args.workload)
-    dtype = torch.bfloat16 if wl.dtype == "bf16" else torch.float32
-    esize = 2 if wl.dtype == "bf16" else 4
-    flat, params = I.init_params_flat(specs, dtype, "cuda", seed=0)
-    plan = es.plan_from_tensors(params)
+    flat, params, plan, esize = param_set(es, args.workload)
     P = plan.numel
     stream = torch.cuda.current_stream()
     sh = stream.cuda_stream
@@ -980,8 +1131,12 @@ class E2ELoop:
         for e in ends:
             lo = params[start].data_ptr() - flat.data_ptr()
             hi = params[e - 1].data_ptr() - flat.data_ptr() + params[e - 1].numel() * esize
-            self.spans.append((lo // esize, hi // esize,
-                               es.es_plan_create(segs_all[start:e], plan.dtype, params[start:e])))
+            if plan.scales is not None:
+                group = es.es_plan_create_scaled(segs_all[start:e], plan.scales[start:e],
+                                                 plan.dtype, params[start:e])
+            else:
+                group = es.es_plan_create(segs_all[start:e], plan.dtype, params[start:e])
+            self.spans.append((lo // esize, hi // esize, group))
             start = e
 
     def step(self, t, record=None):
@@ -1107,19 +1262,25 @@ def oracle_generation(workload: str, n: int, sigma: float, lo: int, count: int, 
     wl = I.WORKLOADS[workload]
     g = np.arange(lo, lo + count, dtype=np.uint64)
     theta32 = I.normal_f32(g.size, lo, 0.02)
-    dt = "bf16" if wl.dtype == "bf16" else "f32"
+    dt = wl.dtype
+    scale = 1.0
     if dt == "bf16":
         import torch
         theta = torch.from_numpy(theta32).to(torch.bfloat16).view(torch.int16).numpy().view(np.uint16)
+    elif dt == "e4m3":
+        import torch
+        scale = float(np.float32(np.abs(theta32).max() / 448.0))
+        theta = torch.from_numpy(theta32 / np.float32(scale)).to(torch.float8_e4m3fn) \
+            .view(torch.uint8).numpy().copy()
     else:
         theta = theta32
     seeds, rewards = generation_inputs(wl, step, n)
     t0 = time.perf_counter()
     for i in range(n):
-        theta = O.perturb(theta, g, int(seeds[i]), sigma, dt)
-        theta = O.restore(theta, g, int(seeds[i]), sigma, dt)
+        theta = O.perturb(theta, g, int(seeds[i]), sigma, dt, scale)
+        theta = O.restore(theta, g, int(seeds[i]), sigma, dt, scale)
     coeffs = O.update_coeffs(O.zscore(rewards), wl.alpha, sigma, 0)
-    theta = O.update(theta, g, seeds, coeffs, dt)
+    theta = O.update(theta, g, seeds, coeffs, dt, scale)
     return time.perf_counter() - t0, g.size
 
 
@@ -1203,7 +1364,11 @@ def run_reference(args, rank, world):
         return
     wl = I.WORKLOADS[args.workload]
     n = args.population or wl.population
-    sigma = float(np.float32(wl.sigma))
+    # the sigma the GPU line reports: the cosine schedule at the first timed step
+    # (the oracle's schedule, equal to the library's to 1e-15)
+    from oracle import oracle as O
+    sigma = float(np.float32(O.sigma_cosine(wl.sigma, SIGMA_FINAL.get(args.workload, wl.sigma),
+                                            args.warmup, SCHEDULE_T)))
     cores = host_cores()
     per_worker = 1 << 17
     pool = OraclePool(cores)
@@ -1250,6 +1415,8 @@ def main():
             run_antithetic(args, rank, world, dist)
         elif args.generator:
             run_generator(args, rank, world, dist)
+        elif args.pipe_peaks:
+            run_pipe_peaks(args, rank, world, dist)
         else:
             run_ours(args, rank, world, dist)
     finally:

@@ -81,8 +81,17 @@ typedef enum {
   ES_ERR_WRONG_DEVICE = 8    /* plan used while another device is current     */
 } es_status_t;
 
-/* Storage type of the parameters. Arithmetic is fp32 in every case. */
-typedef enum { ES_BF16 = 0, ES_FP32 = 1 } es_dtype_t;
+/*
+ * Storage type of the parameters. Arithmetic is fp32 in every case.
+ * ES_FP8_E4M3 stores each element as an 8-bit E4M3 float (OCP 8-bit floating
+ * point: 4 exponent bits with bias 7, 3 mantissa bits, subnormals, no
+ * infinities, largest finite value 448) times a scale per segment
+ * (es_plan_create_scaled); results are rounded to the nearest E4M3 value,
+ * ties to even, saturating at +-448. The paper leaves ES on quantized weights
+ * as future work (App. A.2); this storage type changes only the grid the
+ * parameters are rounded to, not the step.
+ */
+typedef enum { ES_BF16 = 0, ES_FP32 = 1, ES_FP8_E4M3 = 2 } es_dtype_t;
 
 /* Scale of the update coefficients (es_update_coeffs). */
 typedef enum {
@@ -126,6 +135,22 @@ typedef struct es_plan* es_plan_t;
  */
 es_status_t es_plan_create(const es_segment_t* segs, int nseg, es_dtype_t dtype,
                            es_plan_t* out);
+
+/*
+ * A plan whose segments carry one scale each: element k of segment j has the
+ * value scales[j] * stored[k]. For ES_FP8_E4M3 storage, whose range and
+ * spacing are fixed, the scale places a tensor's values on the E4M3 grid (a
+ * per-tensor scale such as max|w| / 448). Every device entry point then works
+ * on the scaled values: a perturb adds sigma * eps to scales[j] * stored[k]
+ * and stores the nearest E4M3 value of the result divided by scales[j].
+ * scales is a host array of nseg finite values > 0 whose reciprocals are
+ * finite; it may be freed after the call. es_plan_create on ES_FP8_E4M3
+ * segments uses scale 1 for every segment. Only ES_FP8_E4M3 takes scales.
+ * Segment rules and errors as es_plan_create, and ES_ERR_INVALID_ARG for a
+ * NULL, non-finite or non-positive scale or another dtype.
+ */
+es_status_t es_plan_create_scaled(const es_segment_t* segs, const float* scales, int nseg,
+                                  es_dtype_t dtype, es_plan_t* out);
 
 /* Frees the plan's device table (synchronises the device). NULL is a no-op. */
 es_status_t es_plan_destroy(es_plan_t plan);
@@ -337,8 +362,13 @@ es_status_t es_fold_antithetic(const double* rhat_pos, const double* rhat_neg,
  *     that overlap on the GPU (on different streams, or from several host
  *     threads without ordering) race on that array and must not be issued.
  *   - The first call on each device looks up the array's device address
- *     (cudaGetSymbolAddress) with that device current; make that first call
- *     before any stream capture.
+ *     (cudaGetSymbolAddress) with that device current and keeps it for that
+ *     device's context (after a device reset the next call looks it up
+ *     again); make that first call before any stream capture.
+ *   - A call on a stream that is being captured is refused with
+ *     ES_ERR_INVALID_ARG before anything is copied or launched: the table is
+ *     copied from the call's own stack, which a recorded copy would read again
+ *     long after the call has returned.
  * Errors: ES_ERR_INVALID_ARG, ES_ERR_ALIGNMENT, ES_ERR_OVERLAP,
  * ES_ERR_NONFINITE, ES_ERR_CUDA.
  */

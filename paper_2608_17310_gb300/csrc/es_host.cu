@@ -22,7 +22,8 @@ struct es_plan {
   int nseg;
   uint64_t numel;
   uint64_t total_tiles;
-  esopt::SegDesc* d_segs;
+  esopt::SegDesc* d_segs;    // one allocation: the table, then (FP8) the
+  float* d_inv_scale;        // reciprocal scales, or NULL
 };
 
 namespace {
@@ -46,7 +47,7 @@ es_status_t cuda_fail(cudaError_t err, const char* what) {
   return fail(ES_ERR_CUDA, "%s: %s (%s)", what, cudaGetErrorName(err), cudaGetErrorString(err));
 }
 
-size_t dtype_size(es_dtype_t dt) { return dt == ES_BF16 ? 2u : 4u; }
+size_t dtype_size(es_dtype_t dt) { return esopt::dtype_bytes(dt); }
 
 es_status_t check_plan_device(const es_plan* plan) {
   int cur = -1;
@@ -69,7 +70,7 @@ es_status_t check_device_buffer(const void* p, const char* what) {
 }
 
 esopt::PlanView view(const es_plan* plan) {
-  return esopt::PlanView{plan->d_segs, plan->total_tiles, plan->dtype};
+  return esopt::PlanView{plan->d_segs, plan->total_tiles, plan->dtype, plan->d_inv_scale};
 }
 
 es_status_t check_update_inputs(es_plan_t plan, const uint64_t* seeds, const float* coeffs, int n,
@@ -139,15 +140,17 @@ es_status_t record_status(es_status_t status, const char* message) {
 }
 }  // namespace esopt
 
-extern "C" {
+namespace {
 
-es_status_t es_plan_create(const es_segment_t* segs, int nseg, es_dtype_t dtype,
-                           es_plan_t* out) {
+// es_plan_create and es_plan_create_scaled: `scales` is NULL (scale 1 for
+// every segment) or nseg checked positive scales, FP8 only.
+es_status_t create_plan(const es_segment_t* segs, const float* scales, int nseg,
+                        es_dtype_t dtype, es_plan_t* out) {
   if (out == nullptr) return fail(ES_ERR_INVALID_ARG, "es_plan_create: out is NULL");
   *out = nullptr;
   if (segs == nullptr || nseg < 1)
     return fail(ES_ERR_INVALID_ARG, "es_plan_create: need at least one segment");
-  if (dtype != ES_BF16 && dtype != ES_FP32)
+  if (dtype != ES_BF16 && dtype != ES_FP32 && dtype != ES_FP8_E4M3)
     return fail(ES_ERR_INVALID_ARG, "es_plan_create: unknown dtype %d", static_cast<int>(dtype));
   const size_t esize = dtype_size(dtype);
   uint64_t total = 0;
@@ -213,10 +216,21 @@ es_status_t es_plan_create(const es_segment_t* segs, int nseg, es_dtype_t dtype,
     if (!esopt::is_device_memory(segs[k].data, device))
       return fail(ES_ERR_INVALID_ARG, "segment %d: not device memory of the current device %d",
                   k, device);
+  // FP8 segments: the kernels take 1 / scale per segment (1 without scales).
+  std::vector<float> inv;
+  if (dtype == ES_FP8_E4M3) {
+    try {
+      inv.resize(static_cast<size_t>(nseg));
+    } catch (const std::bad_alloc&) {
+      return fail(ES_ERR_NO_MEMORY, "es_plan_create: host allocation failed");
+    }
+    for (int k = 0; k < nseg; ++k) inv[k] = scales ? 1.0f / scales[k] : 1.0f;
+  }
   es_plan* plan = new (std::nothrow) es_plan{};
   if (plan == nullptr) return fail(ES_ERR_NO_MEMORY, "es_plan_create: host allocation failed");
   plan->device = device;
-  const size_t bytes = table.size() * sizeof(esopt::SegDesc);
+  const size_t table_bytes = table.size() * sizeof(esopt::SegDesc);
+  const size_t bytes = table_bytes + inv.size() * sizeof(float);
   err = cudaMalloc(reinterpret_cast<void**>(&plan->d_segs), bytes);
   if (err != cudaSuccess) {
     delete plan;
@@ -224,7 +238,12 @@ es_status_t es_plan_create(const es_segment_t* segs, int nseg, es_dtype_t dtype,
     return fail(err == cudaErrorMemoryAllocation ? ES_ERR_NO_MEMORY : ES_ERR_CUDA,
                 "cudaMalloc(segment table): %s", cudaGetErrorString(err));
   }
-  err = cudaMemcpy(plan->d_segs, table.data(), bytes, cudaMemcpyHostToDevice);
+  err = cudaMemcpy(plan->d_segs, table.data(), table_bytes, cudaMemcpyHostToDevice);
+  if (err == cudaSuccess && !inv.empty()) {
+    plan->d_inv_scale = reinterpret_cast<float*>(reinterpret_cast<char*>(plan->d_segs) + table_bytes);
+    err = cudaMemcpy(plan->d_inv_scale, inv.data(), inv.size() * sizeof(float),
+                     cudaMemcpyHostToDevice);
+  }
   if (err != cudaSuccess) {
     cudaFree(plan->d_segs);
     delete plan;
@@ -236,6 +255,30 @@ es_status_t es_plan_create(const es_segment_t* segs, int nseg, es_dtype_t dtype,
   plan->total_tiles = tiles;
   *out = plan;
   return ok();
+}
+
+}  // namespace
+
+extern "C" {
+
+es_status_t es_plan_create(const es_segment_t* segs, int nseg, es_dtype_t dtype,
+                           es_plan_t* out) {
+  return create_plan(segs, nullptr, nseg, dtype, out);
+}
+
+es_status_t es_plan_create_scaled(const es_segment_t* segs, const float* scales, int nseg,
+                                  es_dtype_t dtype, es_plan_t* out) {
+  if (out != nullptr) *out = nullptr;
+  if (dtype != ES_FP8_E4M3)
+    return fail(ES_ERR_INVALID_ARG, "es_plan_create_scaled: only ES_FP8_E4M3 takes scales");
+  if (scales == nullptr || nseg < 1)
+    return fail(ES_ERR_INVALID_ARG, "es_plan_create_scaled: need one scale per segment");
+  for (int k = 0; k < nseg; ++k)
+    if (!std::isfinite(scales[k]) || !(scales[k] > 0.0f) || !std::isfinite(1.0f / scales[k]))
+      return fail(ES_ERR_INVALID_ARG,
+                  "es_plan_create_scaled: scale %d must be finite and > 0 with a finite "
+                  "reciprocal", k);
+  return create_plan(segs, scales, nseg, dtype, out);
 }
 
 es_status_t es_plan_destroy(es_plan_t plan) {

@@ -12,32 +12,55 @@ namespace esopt {
 
 // Threads per CTA of the streaming kernels.
 constexpr int kBlockThreads = 256;
-// Minimum resident CTAs per SM requested from the compiler (a register cap)
-// for the perturb/restore kernels and for the update kernel; 0 leaves the
-// choice to the compiler.
-#ifndef ES_AXPY_MIN_BLOCKS
-#define ES_AXPY_MIN_BLOCKS 1
+// 16-byte vectors per thread in one tile. A tile (kBlockThreads x
+// kVecsPerThread vectors) is the unit a CTA takes from a plan; tiles never
+// straddle segments.
+constexpr int kVecsPerThread = 4;
+
+// Per kernel kind (one-seed pass, two-seed pass, update): how many of its
+// tile vectors a thread processes at once (the group; each vector is
+// vec_elems / 4 independent Philox chains), and the resident CTAs per SM asked
+// of the compiler (a register cap; 1 leaves registers to the compiler). A
+// smaller group needs fewer registers, so more warps fit on an SM.
+#ifndef ES_AXPY1_GROUP
+#define ES_AXPY1_GROUP 4
+#endif
+#ifndef ES_AXPY1_MIN_BLOCKS
+#define ES_AXPY1_MIN_BLOCKS 1
+#endif
+#ifndef ES_AXPY2_GROUP
+#define ES_AXPY2_GROUP 4
+#endif
+#ifndef ES_AXPY2_MIN_BLOCKS
+#define ES_AXPY2_MIN_BLOCKS 1
+#endif
+#ifndef ES_UPDATE_GROUP
+#define ES_UPDATE_GROUP 4
 #endif
 #ifndef ES_UPDATE_MIN_BLOCKS
-#define ES_UPDATE_MIN_BLOCKS 0
+#define ES_UPDATE_MIN_BLOCKS 1
 #endif
-#if ES_AXPY_MIN_BLOCKS > 0
-#define ES_AXPY_BOUNDS __launch_bounds__(esopt::kBlockThreads, ES_AXPY_MIN_BLOCKS)
-#else
-#define ES_AXPY_BOUNDS __launch_bounds__(esopt::kBlockThreads)
+// Seeds of the update's seed loop issued together (independent generator
+// work per element across seeds; the accumulation stays in ascending order).
+#ifndef ES_SEED_UNROLL
+#define ES_SEED_UNROLL 1
 #endif
-#if ES_UPDATE_MIN_BLOCKS > 0
-#define ES_UPDATE_BOUNDS __launch_bounds__(esopt::kBlockThreads, ES_UPDATE_MIN_BLOCKS)
-#else
-#define ES_UPDATE_BOUNDS __launch_bounds__(esopt::kBlockThreads)
-#endif
-// 16-byte vectors each thread owns per tile. All of them are processed in one
-// pass: the independent Philox chains (ILP) matter more than occupancy here
-// (measured: splitting into passes of 1 or 2 vectors, or 8 vectors per
-// thread, were slower).
-constexpr int kVecsPerThread = 4;
+constexpr int kAxpy1Group = ES_AXPY1_GROUP;
+constexpr int kAxpy2Group = ES_AXPY2_GROUP;
+constexpr int kUpdateGroup = ES_UPDATE_GROUP;
+static_assert(kVecsPerThread % kAxpy1Group == 0 && kVecsPerThread % kAxpy2Group == 0 &&
+                  kVecsPerThread % kUpdateGroup == 0,
+              "groups divide the vectors of a tile");
+constexpr int axpy_min_blocks(bool two) {
+  return (two ? ES_AXPY2_MIN_BLOCKS : ES_AXPY1_MIN_BLOCKS) > 0
+             ? (two ? ES_AXPY2_MIN_BLOCKS : ES_AXPY1_MIN_BLOCKS)
+             : 1;
+}
+constexpr int update_min_blocks() { return ES_UPDATE_MIN_BLOCKS > 0 ? ES_UPDATE_MIN_BLOCKS : 1; }
 // Elements per 16-byte vector, per dtype.
-constexpr int vec_elems(es_dtype_t dt) { return dt == ES_BF16 ? 8 : 4; }
+constexpr int vec_elems(es_dtype_t dt) { return dt == ES_FP8_E4M3 ? 16 : dt == ES_BF16 ? 8 : 4; }
+// Bytes per element, per dtype.
+constexpr size_t dtype_bytes(es_dtype_t dt) { return dt == ES_FP8_E4M3 ? 1u : dt == ES_BF16 ? 2u : 4u; }
 // Elements per tile: a tile is the unit one CTA processes at a time; tiles
 // never straddle segments.
 constexpr uint64_t tile_elems(es_dtype_t dt) {
@@ -78,6 +101,8 @@ struct PlanView {
   const SegDesc* segs;  // device table (nseg + 1 entries)
   uint64_t total_tiles;
   es_dtype_t dtype;
+  // ES_FP8_E4M3: device array of 1 / scale per segment; NULL otherwise
+  const float* inv_scale;
 };
 
 // Kernel launchers (es_kernels.cu). Each returns the launch's cudaError_t.

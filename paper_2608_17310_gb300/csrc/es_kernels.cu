@@ -10,9 +10,12 @@
 // Every element is owned by exactly one thread: no atomics, no shared state
 // between threads except the staged seeds of the update.
 #include <cuda_bf16.h>
+#include <cuda_fp16.h>
+#include <cuda_fp8.h>
 #include <cuda_runtime.h>
 
 #include <cstdint>
+#include <mutex>
 
 #include "es_internal.h"
 #include "es_noise.cuh"
@@ -23,7 +26,7 @@ namespace {
 // 16-byte vector <-> fp32 registers, and single-element access for tails.
 struct Bf16Io {
   static constexpr int kVec = 8;
-  static constexpr int kVecs = kVecsPerThread;
+  static constexpr bool kScaled = false;
   using Scalar = uint16_t;
   __device__ static float to_f32(uint16_t h) { return __uint_as_float(static_cast<uint32_t>(h) << 16); }
   __device__ static uint16_t from_f32(float f) { return __bfloat16_as_ushort(__float2bfloat16_rn(f)); }
@@ -50,7 +53,6 @@ struct Bf16Io {
       f[k + 1] = __uint_as_float(w & 0xFFFF0000u);
     }
   }
-  __device__ static float round_trip1(float f) { return to_f32(from_f32(f)); }
   // The first `rem` (< 8) elements at base[e], the rest zero, as one vector.
   __device__ static uint4 load_partial(const uint16_t* base, uint64_t e, int rem) {
     uint32_t w[4] = {0u, 0u, 0u, 0u};
@@ -69,7 +71,7 @@ struct Bf16Io {
 
 struct F32Io {
   static constexpr int kVec = 4;
-  static constexpr int kVecs = kVecsPerThread;
+  static constexpr bool kScaled = false;
   using Scalar = float;
   __device__ static float to_f32(float f) { return f; }
   __device__ static float from_f32(float f) { return f; }
@@ -83,7 +85,6 @@ struct F32Io {
   }
   template <int M>
   __device__ static void round_trip(float (&)[M]) {}
-  __device__ static float round_trip1(float f) { return f; }
   __device__ static uint4 load_partial(const float* base, uint64_t e, int rem) {
     uint32_t w[4] = {0u, 0u, 0u, 0u};
 #pragma unroll
@@ -98,6 +99,86 @@ struct F32Io {
       if (k < rem) base[e + k] = __uint_as_float(w[k]);
   }
 };
+
+// FP8 E4M3 storage: 16 elements per 16-byte vector, byte k of the vector is
+// element k. Values stay in units of the segment's scale: the kernels multiply
+// the noise by 1 / scale instead (kScaled). Decoding goes through half
+// precision, which holds every E4M3 value exactly; encoding rounds fp32 to the
+// nearest E4M3 value, ties to even, saturating at +-448 (cvt .satfinite).
+struct Fp8Io {
+  static constexpr int kVec = 16;
+  static constexpr bool kScaled = true;
+  using Scalar = uint8_t;
+  __device__ static float2 dec2(uint32_t pair) {
+    const __half2_raw h =
+        __nv_cvt_fp8x2_to_halfraw2(static_cast<__nv_fp8x2_storage_t>(pair & 0xFFFFu), __NV_E4M3);
+    return __half22float2(__half2(h));
+  }
+  __device__ static uint32_t enc2(float lo, float hi) {
+    return static_cast<uint32_t>(__nv_cvt_float2_to_fp8x2(make_float2(lo, hi), __NV_SATFINITE,
+                                                          __NV_E4M3));
+  }
+  __device__ static float to_f32(uint8_t c) {
+    return __half2float(__half(__nv_cvt_fp8_to_halfraw(static_cast<__nv_fp8_storage_t>(c),
+                                                       __NV_E4M3)));
+  }
+  __device__ static uint8_t from_f32(float f) {
+    return static_cast<uint8_t>(__nv_cvt_float_to_fp8(f, __NV_SATFINITE, __NV_E4M3));
+  }
+  __device__ static void unpack(const uint4& v, float (&f)[16]) {
+    const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+      const float2 a = dec2(w[k]), b = dec2(w[k] >> 16);
+      f[4 * k + 0] = a.x; f[4 * k + 1] = a.y; f[4 * k + 2] = b.x; f[4 * k + 3] = b.y;
+    }
+  }
+  __device__ static uint4 pack(const float (&f)[16]) {
+    uint32_t w[4];
+#pragma unroll
+    for (int k = 0; k < 4; ++k)
+      w[k] = enc2(f[4 * k + 0], f[4 * k + 1]) | (enc2(f[4 * k + 2], f[4 * k + 3]) << 16);
+    return make_uint4(w[0], w[1], w[2], w[3]);
+  }
+  template <int M>
+  __device__ static void round_trip(float (&f)[M]) {
+#pragma unroll
+    for (int k = 0; k < M; k += 2) {
+      const float2 r = dec2(enc2(f[k], f[k + 1]));
+      f[k] = r.x;
+      f[k + 1] = r.y;
+    }
+  }
+  // The first `rem` (< 16) elements at base[e], the rest zero, as one vector.
+  __device__ static uint4 load_partial(const uint8_t* base, uint64_t e, int rem) {
+    uint32_t w[4] = {0u, 0u, 0u, 0u};
+#pragma unroll
+    for (int k = 0; k < 16; ++k)
+      if (k < rem) w[k >> 2] |= static_cast<uint32_t>(base[e + k]) << (8 * (k & 3));
+    return make_uint4(w[0], w[1], w[2], w[3]);
+  }
+  __device__ static void store_partial(uint8_t* base, uint64_t e, int rem, const uint4& v) {
+    const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+    for (int k = 0; k < 16; ++k)
+      if (k < rem) base[e + k] = static_cast<uint8_t>(w[k >> 2] >> (8 * (k & 3)));
+  }
+};
+
+// Vectors a thread processes at once for a kernel kind's group g: FP8 vectors
+// hold twice the elements of bf16 ones, so they go half as many at a time.
+template <class Io>
+__host__ __device__ constexpr int group_for(int g) {
+  return Io::kVec > 8 ? (g > 1 ? g / 2 : 1) : g;
+}
+
+// theta + acc in storage units: acc is in parameter units, so a scaled
+// segment takes acc / scale (one fused multiply-add with 1 / scale).
+template <class Io>
+__device__ __forceinline__ float add_acc(float theta, float acc, float inv_scale) {
+  if constexpr (Io::kScaled) return fmaf(acc, inv_scale, theta);
+  else return theta + acc;
+}
 
 // Philox words of block j for one seed. TileGen serves the blocks of a tile
 // that share the high counter word (per-tile constants, see philox_tile);
@@ -220,12 +301,13 @@ __device__ __forceinline__ TileRef<Io> tile_ref(const SegDesc* __restrict__ segs
 }
 
 // One tile of the perturb/restore pass (kTwo: fused restore + perturb; kSame:
-// both steps use one seed, whose noise is generated once). Each thread loads
-// its vectors, adds the noise and stores them, all in one pass.
-template <class Io, bool kTwo, bool kSame, bool kUniformHi>
+// both steps use one seed, whose noise is generated once). Each thread takes
+// its kVecsPerThread vectors G at a time: loads them, adds the noise and
+// stores them.
+template <class Io, bool kTwo, bool kSame, bool kUniformHi, int G>
 __device__ __forceinline__ void axpy_tile(const TileRef<Io>& r, PhiloxKey key, float scale,
                                           PhiloxKey key2, float scale2) {
-  constexpr int V = Io::kVec, U = Io::kVecs;
+  constexpr int V = Io::kVec;
   // the two-seed pass is fastest fully packed, the one-seed pass scalar
   constexpr NoiseForm kAxpyForm = kTwo ? NoiseForm::kPacked : NoiseForm::kScalar;
   typename Io::Scalar* const base = r.base;
@@ -233,40 +315,44 @@ __device__ __forceinline__ void axpy_tile(const TileRef<Io>& r, PhiloxKey key, f
   const uint32_t j_hi = static_cast<uint32_t>((index_base + t0) >> 34);
   const auto gen = make_gen<kUniformHi>(key, j_hi);
   const auto gen2 = make_gen<kUniformHi && kTwo && !kSame>(key2, j_hi);
-  uint4 v[U];
+#pragma unroll 1
+  for (int u0 = 0; u0 < kVecsPerThread; u0 += G) {
+    uint4 v[G];
 #pragma unroll
-  for (int u = 0; u < U; ++u) {
-    const uint64_t e = t0 + static_cast<uint64_t>(u * kBlockThreads + threadIdx.x) * V;
-    if (e + V <= numel) v[u] = *reinterpret_cast<const uint4*>(base + e);
-  }
-#pragma unroll
-  for (int u = 0; u < U; ++u) {
-    const uint64_t e = t0 + static_cast<uint64_t>(u * kBlockThreads + threadIdx.x) * V;
-    if (e >= numel) continue;
-    const bool full = e + V <= numel;
-    const int rem = full ? V : static_cast<int>(numel - e);
-    float f[V];
-    if (full) {
-      Io::unpack(v[u], f);
-    } else {  // ragged end of a segment
-#pragma unroll
-      for (int k = 0; k < V; ++k) f[k] = k < rem ? Io::to_f32(base[e + k]) : 0.0f;
+    for (int u = 0; u < G; ++u) {
+      const uint64_t e = t0 + static_cast<uint64_t>((u0 + u) * kBlockThreads + threadIdx.x) * V;
+      v[u] = make_uint4(0u, 0u, 0u, 0u);
+      if (e + V <= numel) v[u] = *reinterpret_cast<const uint4*>(base + e);
     }
-    if (kSame) {
-      add_scaled_noise_twice<Io, V>(gen, index_base + e, scale, scale2, f);
-    } else {
-      add_scaled_noise<kAxpyForm, V>(gen, index_base + e, scale, f);
-      if (kTwo) {
-        Io::round_trip(f);
-        add_scaled_noise<kAxpyForm, V>(gen2, index_base + e, scale2, f);
+#pragma unroll
+    for (int u = 0; u < G; ++u) {
+      const uint64_t e = t0 + static_cast<uint64_t>((u0 + u) * kBlockThreads + threadIdx.x) * V;
+      if (e >= numel) continue;
+      const bool full = e + V <= numel;
+      const int rem = full ? V : static_cast<int>(numel - e);
+      float f[V];
+      if (full) {
+        Io::unpack(v[u], f);
+      } else {  // ragged end of a segment
+#pragma unroll
+        for (int k = 0; k < V; ++k) f[k] = k < rem ? Io::to_f32(base[e + k]) : 0.0f;
       }
-    }
-    if (full) {
-      *reinterpret_cast<uint4*>(base + e) = Io::pack(f);
-    } else {
+      if (kSame) {
+        add_scaled_noise_twice<Io, V>(gen, index_base + e, scale, scale2, f);
+      } else {
+        add_scaled_noise<kAxpyForm, V>(gen, index_base + e, scale, f);
+        if (kTwo) {
+          Io::round_trip(f);
+          add_scaled_noise<kAxpyForm, V>(gen2, index_base + e, scale2, f);
+        }
+      }
+      if (full) {
+        *reinterpret_cast<uint4*>(base + e) = Io::pack(f);
+      } else {
 #pragma unroll
-      for (int k = 0; k < V; ++k)
-        if (k < rem) base[e + k] = Io::from_f32(f[k]);
+        for (int k = 0; k < V; ++k)
+          if (k < rem) base[e + k] = Io::from_f32(f[k]);
+      }
     }
   }
 }
@@ -276,41 +362,53 @@ __device__ __forceinline__ void axpy_tile(const TileRef<Io>& r, PhiloxKey key, f
 // after the first result has been rounded to the storage type exactly as a
 // separate launch would store it (restore of one member fused with the
 // perturb of the next).
+// For a scaled storage type (FP8) the noise is added in units of the
+// segment's scale: scale * inv_scale[segment].
 template <class Io, bool kTwo, bool kSame>
-__global__ void ES_AXPY_BOUNDS
-axpy_noise_kernel(const SegDesc* __restrict__ segs, uint64_t total_tiles, PhiloxKey key,
-                  float scale, PhiloxKey key2, float scale2) {
+__global__ void __launch_bounds__(kBlockThreads, axpy_min_blocks(kTwo))
+axpy_noise_kernel(const SegDesc* __restrict__ segs, const float* __restrict__ inv_scale,
+                  uint64_t total_tiles, PhiloxKey key, float scale, PhiloxKey key2,
+                  float scale2) {
   constexpr uint64_t kTile = static_cast<uint64_t>(kBlockThreads) * kVecsPerThread * Io::kVec;
+  constexpr int G = group_for<Io>(kTwo ? kAxpy2Group : kAxpy1Group);
   int seg = 0;
   for (uint64_t tile = blockIdx.x; tile < total_tiles; tile += gridDim.x) {
     const TileRef<Io> cur = tile_ref<Io>(segs, seg, tile, kTile);
+    float s1 = scale, s2 = scale2;
+    if constexpr (Io::kScaled) {
+      const float inv = inv_scale[seg];
+      s1 *= inv;
+      s2 *= inv;
+    }
     if (uniform_hi(cur.index_base, cur.t0, kTile, cur.numel))
-      axpy_tile<Io, kTwo, kSame, true>(cur, key, scale, key2, scale2);
+      axpy_tile<Io, kTwo, kSame, true, G>(cur, key, s1, key2, s2);
     else
-      axpy_tile<Io, kTwo, kSame, false>(cur, key, scale, key2, scale2);
+      axpy_tile<Io, kTwo, kSame, false, G>(cur, key, s1, key2, s2);
   }
 }
 
 // One tile of a single-generation update (es_update; with kPerturb also the
 // trailing perturb of es_update_perturb): acc = sum_i c_i eps_i (fp32,
 // ascending i), then theta + acc rounded once (then + pscale * eps_pseed,
-// rounded again); theta read and written once.
-template <class Io, bool kUniformHi, bool kPerturb>
+// rounded again); theta read and written once. Vectors G at a time.
+template <class Io, bool kUniformHi, bool kPerturb, int G>
 __device__ __forceinline__ void update_tile_single(typename Io::Scalar* base, uint64_t numel,
                                                    uint64_t index_base, uint64_t t0,
                                                    const UpdateArgs& args, const PhiloxKey* s_key,
-                                                   const float* s_coeff) {
+                                                   const float* s_coeff, float inv) {
   constexpr int V = Io::kVec;
-  constexpr int G = Io::kVecs;
+  constexpr int kUnroll = ES_SEED_UNROLL;
   const uint32_t j_hi = static_cast<uint32_t>((index_base + t0) >> 34);
   const int n = args.n;
+  const float pscale = Io::kScaled ? args.pscale * inv : args.pscale;
   const auto pgen = make_gen<kUniformHi && kPerturb>(PhiloxKey{args.pkey[0], args.pkey[1]}, j_hi);
-  {
-    constexpr int u0 = 0;
+#pragma unroll 1
+  for (int u0 = 0; u0 < kVecsPerThread; u0 += G) {
     uint4 v[G];
 #pragma unroll
     for (int q = 0; q < G; ++q) {
       const uint64_t e = t0 + static_cast<uint64_t>((u0 + q) * kBlockThreads + threadIdx.x) * V;
+      v[q] = make_uint4(0u, 0u, 0u, 0u);
       if (e + V <= numel) v[q] = *reinterpret_cast<const uint4*>(base + e);
     }
     float acc[G][V];
@@ -318,7 +416,7 @@ __device__ __forceinline__ void update_tile_single(typename Io::Scalar* base, ui
     for (int q = 0; q < G; ++q)
 #pragma unroll
       for (int k = 0; k < V; ++k) acc[q][k] = 0.0f;
-#pragma unroll 1
+#pragma unroll kUnroll
     for (int i = 0; i < n; ++i) {
       const auto gen = make_gen<kUniformHi>(s_key[i], j_hi);
       const float c = s_coeff[i];
@@ -343,10 +441,10 @@ __device__ __forceinline__ void update_tile_single(typename Io::Scalar* base, ui
         for (int k = 0; k < V; ++k) f[k] = k < rem ? Io::to_f32(base[e + k]) : 0.0f;
       }
 #pragma unroll
-      for (int k = 0; k < V; ++k) f[k] = f[k] + acc[q][k];
+      for (int k = 0; k < V; ++k) f[k] = add_acc<Io>(f[k], acc[q][k], inv);
       if (kPerturb) {
         Io::round_trip(f);
-        add_scaled_noise<NoiseForm::kPackedFma, V>(pgen, index_base + e, args.pscale, f);
+        add_scaled_noise<NoiseForm::kPackedFma, V>(pgen, index_base + e, pscale, f);
       }
       if (full) {
         *reinterpret_cast<uint4*>(base + e) = Io::pack(f);
@@ -363,20 +461,23 @@ __device__ __forceinline__ void update_tile_single(typename Io::Scalar* base, ui
 // form; generation g adds acc_g = sum_{i in g} c_i eps_i (fp32, ascending i)
 // and rounds once, exactly as a separate launch per generation would store it;
 // an optional trailing perturb step follows. Theta is read and written once.
-template <class Io, bool kUniformHi>
+// Vectors G at a time; lanes past the segment's end hold zeros and are never
+// stored.
+template <class Io, bool kUniformHi, int G>
 __device__ __forceinline__ void update_tile(typename Io::Scalar* base, uint64_t numel,
                                             uint64_t index_base, uint64_t t0,
                                             const UpdateArgs& args, const PhiloxKey* s_key,
-                                            const float* s_coeff, const uint16_t* s_gen_end) {
+                                            const float* s_coeff, const uint16_t* s_gen_end,
+                                            float inv) {
   constexpr int V = Io::kVec;
-  constexpr int G = Io::kVecs;
   const uint32_t j_hi = static_cast<uint32_t>((index_base + t0) >> 34);
-  {
-    constexpr int u0 = 0;
+#pragma unroll 1
+  for (int u0 = 0; u0 < kVecsPerThread; u0 += G) {
     uint4 v[G];
 #pragma unroll
     for (int q = 0; q < G; ++q) {
       const uint64_t e = t0 + static_cast<uint64_t>((u0 + q) * kBlockThreads + threadIdx.x) * V;
+      v[q] = make_uint4(0u, 0u, 0u, 0u);
       if (e + V <= numel)
         v[q] = *reinterpret_cast<const uint4*>(base + e);
       else if (e < numel)
@@ -407,7 +508,7 @@ __device__ __forceinline__ void update_tile(typename Io::Scalar* base, uint64_t 
         float f[V];
         Io::unpack(v[q], f);
 #pragma unroll
-        for (int k = 0; k < V; ++k) f[k] = f[k] + acc[q][k];
+        for (int k = 0; k < V; ++k) f[k] = add_acc<Io>(f[k], acc[q][k], inv);
         v[q] = Io::pack(f);
       }
     }
@@ -419,7 +520,8 @@ __device__ __forceinline__ void update_tile(typename Io::Scalar* base, uint64_t 
         if (e >= numel) continue;
         float f[V];
         Io::unpack(v[q], f);
-        add_scaled_noise<NoiseForm::kPackedFma, V>(gen, index_base + e, args.pscale, f);
+        add_scaled_noise<NoiseForm::kPackedFma, V>(gen, index_base + e,
+                                                   Io::kScaled ? args.pscale * inv : args.pscale, f);
         v[q] = Io::pack(f);
       }
     }
@@ -440,10 +542,11 @@ __device__ __forceinline__ void update_tile(typename Io::Scalar* base, uint64_t 
 // kSingle: one generation (update_tile_single, with a trailing perturb when
 // kPerturb); otherwise the general form (update_tile).
 template <class Io, bool kSingle, bool kPerturb>
-__global__ void ES_UPDATE_BOUNDS
-update_kernel(const SegDesc* __restrict__ segs, uint64_t total_tiles,
-              const __grid_constant__ UpdateArgs args) {
+__global__ void __launch_bounds__(kBlockThreads, update_min_blocks())
+update_kernel(const SegDesc* __restrict__ segs, const float* __restrict__ inv_scale,
+              uint64_t total_tiles, const __grid_constant__ UpdateArgs args) {
   constexpr uint64_t kTile = static_cast<uint64_t>(kBlockThreads) * kVecsPerThread * Io::kVec;
+  constexpr int G = group_for<Io>(kUpdateGroup);
   using S = typename Io::Scalar;
   __shared__ PhiloxKey s_key[ES_MAX_SEEDS];
   __shared__ float s_coeff[ES_MAX_SEEDS];
@@ -463,16 +566,21 @@ update_kernel(const SegDesc* __restrict__ segs, uint64_t total_tiles,
     const uint64_t index_base = d->index_base;
     const uint64_t t0 = (tile - d->tile_begin) * kTile;
     const bool uhi = uniform_hi(index_base, t0, kTile, numel);
+    const float inv = Io::kScaled ? inv_scale[seg] : 1.0f;
     if constexpr (kSingle) {
       if (uhi)
-        update_tile_single<Io, true, kPerturb>(base, numel, index_base, t0, args, s_key, s_coeff);
+        update_tile_single<Io, true, kPerturb, G>(base, numel, index_base, t0, args, s_key,
+                                                  s_coeff, inv);
       else
-        update_tile_single<Io, false, kPerturb>(base, numel, index_base, t0, args, s_key, s_coeff);
+        update_tile_single<Io, false, kPerturb, G>(base, numel, index_base, t0, args, s_key,
+                                                   s_coeff, inv);
     } else {
       if (uhi)
-        update_tile<Io, true>(base, numel, index_base, t0, args, s_key, s_coeff, s_gen_end);
+        update_tile<Io, true, G>(base, numel, index_base, t0, args, s_key, s_coeff, s_gen_end,
+                                 inv);
       else
-        update_tile<Io, false>(base, numel, index_base, t0, args, s_key, s_coeff, s_gen_end);
+        update_tile<Io, false, G>(base, numel, index_base, t0, args, s_key, s_coeff, s_gen_end,
+                                  inv);
     }
   }
 }
@@ -560,34 +668,65 @@ box_muller_kernel(const uint2* __restrict__ words, uint64_t npairs, float2* __re
   }
 }
 
-// Persistent grid: every SM filled to the kernel's occupancy, never more
-// CTAs than tiles.
-template <class K>
-int persistent_grid(K kernel, uint64_t work_items) {
-  int dev = 0, sms = 0, per_sm = 0;
-  cudaGetDevice(&dev);
+// Resident CTAs of one kernel on one device (SMs x CTAs per SM), looked up
+// with the occupancy calculator on the kernel's first launch on that device
+// and kept, so later launches make no query beyond cudaGetDevice.
+struct GridEntry {
+  const void* kernel;
+  int device;
+  int ctas;
+};
+constexpr int kGridCacheSize = 128;
+std::mutex g_grid_mutex;
+GridEntry g_grid_cache[kGridCacheSize];
+int g_grid_used = 0;
+
+int resident_ctas(const void* kernel, int dev) {
+  {
+    std::lock_guard<std::mutex> lock(g_grid_mutex);
+    for (int k = 0; k < g_grid_used; ++k)
+      if (g_grid_cache[k].kernel == kernel && g_grid_cache[k].device == dev)
+        return g_grid_cache[k].ctas;
+  }
+  int sms = 0, per_sm = 0;
   cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
   cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kernel, kBlockThreads, 0);
   if (sms < 1) sms = 1;
   if (per_sm < 1) per_sm = 1;
-  uint64_t grid = static_cast<uint64_t>(sms) * per_sm;
+  const int ctas = sms * per_sm;
+  std::lock_guard<std::mutex> lock(g_grid_mutex);
+  if (g_grid_used < kGridCacheSize) g_grid_cache[g_grid_used++] = GridEntry{kernel, dev, ctas};
+  return ctas;
+}
+
+// Persistent grid: every SM filled to the kernel's occupancy, never more
+// CTAs than tiles.
+template <class K>
+int persistent_grid(K kernel, uint64_t work_items) {
+  int dev = 0;
+  cudaGetDevice(&dev);
+  uint64_t grid = static_cast<uint64_t>(resident_ctas(reinterpret_cast<const void*>(kernel), dev));
   if (work_items < grid) grid = work_items;
   return grid < 1 ? 1 : static_cast<int>(grid);
+}
+
+template <class Io, bool kTwo, bool kSame>
+cudaError_t launch_axpy_io(const PlanView& plan, PhiloxKey key, float scale, PhiloxKey key2,
+                           float scale2, cudaStream_t stream) {
+  auto k = axpy_noise_kernel<Io, kTwo, kSame>;
+  k<<<persistent_grid(k, plan.total_tiles), kBlockThreads, 0, stream>>>(
+      plan.segs, plan.inv_scale, plan.total_tiles, key, scale, key2, scale2);
+  return cudaGetLastError();
 }
 
 template <bool kTwo, bool kSame>
 cudaError_t launch_axpy(const PlanView& plan, PhiloxKey key, float scale, PhiloxKey key2,
                         float scale2, cudaStream_t stream) {
-  if (plan.dtype == ES_BF16) {
-    auto k = axpy_noise_kernel<Bf16Io, kTwo, kSame>;
-    k<<<persistent_grid(k, plan.total_tiles), kBlockThreads, 0, stream>>>(
-        plan.segs, plan.total_tiles, key, scale, key2, scale2);
-  } else {
-    auto k = axpy_noise_kernel<F32Io, kTwo, kSame>;
-    k<<<persistent_grid(k, plan.total_tiles), kBlockThreads, 0, stream>>>(
-        plan.segs, plan.total_tiles, key, scale, key2, scale2);
-  }
-  return cudaGetLastError();
+  if (plan.dtype == ES_BF16)
+    return launch_axpy_io<Bf16Io, kTwo, kSame>(plan, key, scale, key2, scale2, stream);
+  if (plan.dtype == ES_FP8_E4M3)
+    return launch_axpy_io<Fp8Io, kTwo, kSame>(plan, key, scale, key2, scale2, stream);
+  return launch_axpy_io<F32Io, kTwo, kSame>(plan, key, scale, key2, scale2, stream);
 }
 
 }  // namespace
@@ -611,14 +750,15 @@ template <class Io>
 cudaError_t launch_update_io(const PlanView& plan, const UpdateArgs& args, cudaStream_t stream) {
   auto k = update_kernel<Io, false, false>;
   if (args.n_gen == 1) k = args.perturb ? update_kernel<Io, true, true> : update_kernel<Io, true, false>;
-  k<<<persistent_grid(k, plan.total_tiles), kBlockThreads, 0, stream>>>(plan.segs, plan.total_tiles,
-                                                                          args);
+  k<<<persistent_grid(k, plan.total_tiles), kBlockThreads, 0, stream>>>(
+      plan.segs, plan.inv_scale, plan.total_tiles, args);
   return cudaGetLastError();
 }
 
 cudaError_t launch_update(const PlanView& plan, const UpdateArgs& args, cudaStream_t stream) {
-  return plan.dtype == ES_BF16 ? launch_update_io<Bf16Io>(plan, args, stream)
-                               : launch_update_io<F32Io>(plan, args, stream);
+  if (plan.dtype == ES_BF16) return launch_update_io<Bf16Io>(plan, args, stream);
+  if (plan.dtype == ES_FP8_E4M3) return launch_update_io<Fp8Io>(plan, args, stream);
+  return launch_update_io<F32Io>(plan, args, stream);
 }
 
 cudaError_t launch_noise_bits(uint64_t seed, uint64_t block_base, uint64_t nblocks,

@@ -3,6 +3,7 @@
 // memory es_plan_create obtains with cudaMalloc), the segment table is copied
 // on every call into a fixed array of static device memory that belongs to
 // this library module.
+#include <cuda.h>
 #include <cuda_runtime.h>
 
 #include <algorithm>
@@ -26,13 +27,52 @@ __device__ __align__(256) SegDesc g_noalloc_table[ES_STATIC_MAX_SEGMENTS + 1];
 constexpr int kMaxDevices = 64;
 std::mutex g_setup_mutex;
 SegDesc* g_table_address[kMaxDevices] = {};
+// Id of the context the cached address belongs to (0: unknown). A device
+// reset destroys the context and the module loaded into it; the next context
+// gets a new id, and the address is looked up again.
+unsigned long long g_table_context[kMaxDevices] = {};
 
-// Device address of g_noalloc_table on `device` (which is current). In host
+using CtxGetCurrentFn = CUresult (*)(CUcontext*);
+using CtxGetIdFn = CUresult (*)(CUcontext, unsigned long long*);
+
+// Id of the calling thread's current context, or 0 if the driver does not
+// provide one. The driver functions are found at run time, so the library does
+// not link against the driver library.
+unsigned long long current_context_id() {
+  static CtxGetCurrentFn get_current = nullptr;
+  static CtxGetIdFn get_id = nullptr;
+  static bool looked_up = false;
+  if (!looked_up) {
+    looked_up = true;
+    void* fn = nullptr;
+    cudaDriverEntryPointQueryResult q{};
+    if (cudaGetDriverEntryPointByVersion("cuCtxGetCurrent", &fn, 12000, cudaEnableDefault, &q) ==
+            cudaSuccess && q == cudaDriverEntryPointSuccess)
+      get_current = reinterpret_cast<CtxGetCurrentFn>(fn);
+    fn = nullptr;
+    if (cudaGetDriverEntryPointByVersion("cuCtxGetId", &fn, 12000, cudaEnableDefault, &q) ==
+            cudaSuccess && q == cudaDriverEntryPointSuccess)
+      get_id = reinterpret_cast<CtxGetIdFn>(fn);
+    cudaGetLastError();
+  }
+  CUcontext ctx = nullptr;
+  unsigned long long id = 0;
+  if (get_current == nullptr || get_id == nullptr || get_current(&ctx) != CUDA_SUCCESS ||
+      ctx == nullptr || get_id(ctx, &id) != CUDA_SUCCESS)
+    return 0;
+  return id;
+}
+
+// Device address of g_noalloc_table on `device`, which is current. In host
 // code the name g_noalloc_table is only a host-side stand-in, so the address
-// is looked up once per device with cudaGetSymbolAddress and cached.
+// is looked up with cudaGetSymbolAddress once per device (the set-up done by
+// the first call on each device) and cached; it is looked up again when the
+// device's context has changed since (after a device reset), or on every call
+// if the context cannot be identified.
 es_status_t table_address(int device, SegDesc** out) {
   std::lock_guard<std::mutex> lock(g_setup_mutex);
-  if (g_table_address[device] == nullptr) {
+  const unsigned long long ctx = current_context_id();
+  if (g_table_address[device] == nullptr || ctx == 0 || ctx != g_table_context[device]) {
     void* p = nullptr;
     cudaError_t err = cudaGetSymbolAddress(&p, g_noalloc_table);
     if (err != cudaSuccess || p == nullptr) {
@@ -42,6 +82,7 @@ es_status_t table_address(int device, SegDesc** out) {
       return record_status(ES_ERR_CUDA, msg);
     }
     g_table_address[device] = static_cast<SegDesc*>(p);
+    g_table_context[device] = ctx;
   }
   *out = g_table_address[device];
   return ES_OK;
@@ -110,8 +151,24 @@ extern "C" es_status_t es_perturb_noalloc(const es_segment_t* segs, int nseg, es
   }
   table[nseg] = SegDesc{nullptr, 0, 0, tiles};
 
+  // The table is copied from this call's stack; a copy recorded into a graph
+  // would read that memory again at every replay, long after it is gone. So a
+  // stream that is being captured is refused before anything is done.
+  const cudaStream_t s = static_cast<cudaStream_t>(stream);
+  cudaStreamCaptureStatus capture = cudaStreamCaptureStatusNone;
+  cudaError_t err = cudaStreamIsCapturing(s, &capture);
+  if (err != cudaSuccess) {
+    cudaGetLastError();
+    return reject(ES_ERR_CUDA, "es_perturb_noalloc: cudaStreamIsCapturing failed");
+  }
+  if (capture != cudaStreamCaptureStatusNone)
+    return reject(ES_ERR_INVALID_ARG,
+                  "es_perturb_noalloc: the stream is being captured into a CUDA graph; this "
+                  "entry point copies its segment table from host stack memory and is refused "
+                  "on a capturing stream");
+
   int device = -1;
-  cudaError_t err = cudaGetDevice(&device);
+  err = cudaGetDevice(&device);
   if (err != cudaSuccess) return reject(ES_ERR_CUDA, "es_perturb_noalloc: cudaGetDevice failed");
   if (device < 0 || device >= esopt::kMaxDevices)
     return reject(ES_ERR_INVALID_ARG, "es_perturb_noalloc: device ordinal %d >= %d", device,
@@ -127,11 +184,10 @@ extern "C" es_status_t es_perturb_noalloc(const es_segment_t* segs, int nseg, es
   // call, so nothing in it has to start at zero. From pageable host memory
   // the source is staged before cudaMemcpyAsync returns, so `table` may go
   // out of scope; the kernel below is ordered after the copy on `stream`.
-  const cudaStream_t s = static_cast<cudaStream_t>(stream);
   err = cudaMemcpyAsync(d_table, table, (static_cast<size_t>(nseg) + 1) * sizeof(SegDesc),
                         cudaMemcpyHostToDevice, s);
   if (err != cudaSuccess) return reject(ES_ERR_CUDA, "es_perturb_noalloc: copy of the segment table failed");
-  err = esopt::launch_axpy_noise(esopt::PlanView{d_table, tiles, dtype}, seed, sigma, s);
+  err = esopt::launch_axpy_noise(esopt::PlanView{d_table, tiles, dtype, nullptr}, seed, sigma, s);
   if (err != cudaSuccess) return reject(ES_ERR_CUDA, "es_perturb_noalloc: kernel launch failed");
   return esopt::record_status(ES_OK, "");
 }

@@ -39,6 +39,7 @@ ES_ERR_WRONG_DEVICE = 8
 
 ES_BF16 = 0
 ES_FP32 = 1
+ES_FP8_E4M3 = 2
 
 ES_SCALE_PAPER = 0
 ES_SCALE_CANONICAL = 1
@@ -72,6 +73,7 @@ def _load() -> ctypes.CDLL:
     P = ctypes.POINTER
     sigs = {
         "es_plan_create": (i32, [P(es_segment_t), i32, i32, P(vp)]),
+        "es_plan_create_scaled": (i32, [P(es_segment_t), P(f32), i32, i32, P(vp)]),
         "es_plan_destroy": (i32, [vp]),
         "es_plan_numel": (u64, [vp]),
         "es_assign_index_bases": (u64, [P(es_segment_t), i32]),
@@ -155,10 +157,11 @@ class Segment:
 class Plan:
     """Owns an ``es_plan_t``. Keeps the objects that own the memory alive."""
 
-    def __init__(self, handle: int, numel: int, dtype: int, keepalive=()):
+    def __init__(self, handle: int, numel: int, dtype: int, keepalive=(), scales=None):
         self.handle = handle
         self.numel = numel
         self.dtype = dtype
+        self.scales = None if scales is None else [float(x) for x in scales]
         self._keepalive = tuple(keepalive)
 
     def close(self) -> None:
@@ -205,6 +208,20 @@ def es_plan_create(segments: Sequence[Segment], dtype: int, keepalive: Iterable 
     return Plan(handle.value, int(_load().es_plan_numel(handle)), dtype, keepalive)
 
 
+def es_plan_create_scaled(segments: Sequence[Segment], scales, dtype: int,
+                          keepalive: Iterable = ()) -> Plan:
+    """A plan whose segment j holds values scales[j] * stored (ES_FP8_E4M3)."""
+    arr = _seg_array(segments)
+    sc = np.ascontiguousarray(scales, dtype=np.float32)
+    if sc.size != len(segments):
+        raise ValueError("one scale per segment")
+    handle = ctypes.c_void_p()
+    _check(_load().es_plan_create_scaled(arr, sc.ctypes.data_as(ctypes.POINTER(ctypes.c_float)),
+                                         len(segments), dtype, ctypes.byref(handle)),
+           "es_plan_create_scaled")
+    return Plan(handle.value, int(_load().es_plan_numel(handle)), dtype, keepalive, sc)
+
+
 def segments_from_tensors(tensors, index_bases=None):
     """Segments for a list of contiguous CUDA tensors (bases assigned if None)."""
     segs = []
@@ -222,8 +239,10 @@ def segments_from_tensors(tensors, index_bases=None):
     return segs
 
 
-def plan_from_tensors(tensors, index_bases=None) -> Plan:
-    """es_plan_create over torch tensors of one dtype (bf16 or fp32)."""
+def plan_from_tensors(tensors, index_bases=None, scales=None) -> Plan:
+    """es_plan_create over torch tensors of one dtype: bf16, fp32, or FP8 E4M3
+    (torch.float8_e4m3fn, or uint8 holding E4M3 codes), the latter with one
+    scale per tensor (es_plan_create_scaled; all 1 if scales is None)."""
     import torch  # only for the dtype check
     tensors = list(tensors)
     dts = {t.dtype for t in tensors}
@@ -231,9 +250,14 @@ def plan_from_tensors(tensors, index_bases=None) -> Plan:
         dtype = ES_BF16
     elif dts == {torch.float32}:
         dtype = ES_FP32
+    elif dts <= {torch.float8_e4m3fn, torch.uint8}:
+        dtype = ES_FP8_E4M3
     else:
-        raise ValueError(f"all tensors must be bfloat16 or all float32, got {dts}")
-    return es_plan_create(segments_from_tensors(tensors, index_bases), dtype, keepalive=tensors)
+        raise ValueError(f"all tensors must be bfloat16, float32 or FP8 E4M3, got {dts}")
+    segs = segments_from_tensors(tensors, index_bases)
+    if scales is not None:
+        return es_plan_create_scaled(segs, scales, dtype, keepalive=tensors)
+    return es_plan_create(segs, dtype, keepalive=tensors)
 
 
 # --- device entry points ----------------------------------------------------------

@@ -22,6 +22,9 @@ the same shapes):
              heads of dim 128, SwiGLU 17408, vocab 151,936, untied embeddings
              (22,695,777,280 parameters, 579 tensors); N = 30, sigma_0 5e-4,
              Uniform[0,1] rewards
+  qwen4b_fp8 the qwen4b shapes stored as FP8 E4M3 codes with one scale per
+             tensor, amax / 448 of its N(0, 0.02^2) weights (norms: 1 / 448,
+             so 1.0 is the code 448); N = 16, sigma 1e-3, Bernoulli(0.3)
 Weights ~ N(0, 0.02^2), norm weights = 1.
 """
 from __future__ import annotations
@@ -74,7 +77,7 @@ def qwen27b_shapes() -> List[TensorSpec]:
 @dataclass(frozen=True)
 class Workload:
     name: str
-    dtype: str            # "bf16" or "f32"
+    dtype: str            # "bf16", "f32" or "e4m3"
     population: int       # N seeds per update
     sigma: float
     alpha: float
@@ -95,6 +98,11 @@ WORKLOADS = {
     # Gaussian there, so HBM rather than the generator bounds it
     "qwen4b_f32": Workload("qwen4b_f32", "f32", 16, 1e-3, 5e-4, "bernoulli0.3",
                            "Qwen3.5-4B-shaped fp32 (4,022,458,880 params, 326 tensors), N=16"),
+    # the 4B shapes in FP8 E4M3 storage with a scale per tensor (4.0 GB): the
+    # quantized-weight direction of App. A.2 on the config-3 population
+    "qwen4b_fp8": Workload("qwen4b_fp8", "e4m3", 16, 1e-3, 5e-4, "bernoulli0.3",
+                           "Qwen3.5-4B-shaped FP8 E4M3 with per-tensor scales "
+                           "(4,022,458,880 params, 326 tensors), N=16"),
     # profiling case: the 4B shapes cut to 4 layers (about 1.6 GB, larger than L2)
     "qwen4b_4layer": Workload("qwen4b_4layer", "bf16", 16, 1e-3, 5e-4, "bernoulli0.3",
                               "Qwen3.5-4B shapes, 4 layers (792,680,960 params, 38 tensors), N=16"),
@@ -102,7 +110,7 @@ WORKLOADS = {
 
 
 def shapes_for(name: str) -> List[TensorSpec]:
-    if name in ("qwen4b", "qwen4b_f32"):
+    if name in ("qwen4b", "qwen4b_f32", "qwen4b_fp8"):
         return qwen4b_shapes()
     if name == "qwen27b":
         return qwen27b_shapes()
@@ -197,6 +205,33 @@ def init_params_flat(specs: List[TensorSpec], dtype, device, seed: int = 0, std:
             t.normal_(0.0, std, generator=gen)
         views.append(t)
     return flat, views
+
+
+def init_params_flat_e4m3(specs: List[TensorSpec], device, seed: int = 0, std: float = 0.02):
+    """The parameter set as FP8 E4M3 codes in one uint8 allocation: returns
+    (flat buffer, one view per spec, one scale per spec). Each tensor is drawn
+    as in init_params_flat (fp32 here), given the scale amax / 448 (the largest
+    E4M3 magnitude is 448) and stored as the nearest E4M3 codes of w / scale
+    (torch's float8_e4m3fn conversion). Views start at 16-byte offsets."""
+    import torch
+    offs = flat_offsets(specs, align=16)
+    flat = torch.zeros(offs[-1], dtype=torch.uint8, device=device)
+    gen = torch.Generator(device=device)
+    gen.manual_seed(seed)
+    views, scales = [], []
+    for s, o in zip(specs, offs):
+        w = torch.empty(s.numel, dtype=torch.float32, device=device)
+        if s.kind == "norm":
+            w.fill_(1.0)
+        else:
+            w.normal_(0.0, std, generator=gen)
+        scale = float(np.float32(max(float(w.abs().max()), 1e-30) / 448.0))
+        t = flat[o:o + s.numel]
+        t.copy_((w / scale).to(torch.float8_e4m3fn).view(torch.uint8))
+        del w
+        views.append(t)
+        scales.append(scale)
+    return flat, views, scales
 
 
 def sample_offsets(numel: int, n_random: int, seed: int, edge: int = 64) -> np.ndarray:

@@ -47,14 +47,15 @@ def bf16_order(bits):
     return np.where(b & 0x8000, -mag, mag)
 
 
-def _bf16_values(bits):
+def bf16_values(bits):
+    """bf16 bit patterns (uint16) -> float64 values."""
     b = np.asarray(bits, dtype=np.uint16).astype(np.uint32) << 16
     return b.view(np.float32).astype(np.float64)
 
 
 def assert_bf16_within_ulp(got_bits, want_bits, what="", ulps=1, abs_tol=0.0):
     d = np.abs(bf16_order(got_bits) - bf16_order(want_bits))
-    g, w = _bf16_values(got_bits), _bf16_values(want_bits)
+    g, w = bf16_values(got_bits), bf16_values(want_bits)
     ulp = 2.0 ** (np.floor(np.log2(np.maximum(np.maximum(np.abs(g), np.abs(w)), 2.0**-126))) - 7)
     near = np.abs(g - w) <= abs_tol + ulp
     bad = np.nonzero((d > ulps) & ~near)[0]

@@ -227,3 +227,16 @@ def test_last_error_is_per_thread(E):
     for t in threads:
         t.join()
     assert not errors, errors
+
+
+def test_scaled_plan_rejects_bad_scales_before_any_device_call(E):
+    # The scales are checked before the segments are looked at, so this pointer
+    # is never dereferenced.
+    seg = [E.Segment(0x100000, 16, 0)]
+    for bad in (0.0, -1.0, float("nan"), float("inf"), 1e-45):
+        with pytest.raises(E.EsError) as ei:
+            E.es_plan_create_scaled(seg, [bad], E.ES_FP8_E4M3)
+        assert ei.value.status == E.ES_ERR_INVALID_ARG
+    with pytest.raises(E.EsError) as ei:
+        E.es_plan_create_scaled(seg, [1.0], E.ES_BF16)
+    assert ei.value.status == E.ES_ERR_INVALID_ARG

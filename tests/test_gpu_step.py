@@ -5,7 +5,8 @@ import numpy as np
 import pytest
 import torch
 
-from parity import assert_bf16_within_ulp, assert_f32_close, noise_abs_tol
+from parity import (assert_bf16_within_ulp, assert_f32_close, bf16_order, bf16_values,
+                    noise_abs_tol)
 
 pytestmark = pytest.mark.gpu
 
@@ -336,6 +337,138 @@ def test_antithetic_restore_perturb_reuses_one_seed(es, dtype):
         assert torch.equal(_int_view(x), _int_view(y))
     plan_a.close()
     plan_b.close()
+
+
+def _sample(segs, rng, per_seg=2048, edge=64):
+    """Indices into each segment: its first and last `edge` elements plus
+    about `per_seg` random ones (all of a short segment)."""
+    out = []
+    for s in segs:
+        n = s.numel
+        if n <= per_seg + 2 * edge:
+            out.append(np.arange(n))
+            continue
+        idx = np.concatenate([np.arange(edge), np.arange(n - edge, n),
+                              rng.integers(edge, n - edge, size=per_seg)])
+        out.append(np.unique(idx))
+    return out
+
+
+@pytest.mark.parametrize("dtype", ["bf16", "f32"])
+def test_replay_matches_oracle_generation_by_generation(es, oracle, dtype):
+    # The seed log of a run is replayed from the base parameters (App. D.2-D.4):
+    # 400 logged generations. The first 300 have 1..3 seeds, so they share
+    # passes over theta and pass the 256-generation limit of one pass; the
+    # last 100 have 1..8 seeds, so generations of 4 or more get passes of their
+    # own through the single-generation kernel. Some generations and some
+    # coefficients are zero. The oracle applies the same generations one by one
+    # in double precision, rounding to storage after each, from the same start.
+    numels = [9, 8193, 20000, 4096 * 3 + 5]
+    tensors = make_params(dtype, numels, seed=40)
+    plan, segs = build_plan(es, tensors, [8, 2**34 - 1024, 2**36, 2**50])
+    rng = np.random.default_rng(41)
+    counts = np.concatenate([rng.integers(1, 4, size=300), rng.integers(1, 9, size=100)])
+    total = int(counts.sum())
+    seeds = rng.integers(0, 2**63, size=total, dtype=np.uint64)
+    coeffs = (1e-3 * rng.standard_normal(total)).astype(np.float32)
+    coeffs[rng.random(total) < 0.05] = 0.0
+    ends = np.cumsum(counts)
+    starts = ends - counts
+    for gen in (7, 250, 333):
+        coeffs[starts[gen]:ends[gen]] = 0.0
+    pick = _sample(segs, rng)
+    g = indices(segs)
+    state = [host_values(t)[ix] for t, ix in zip(tensors, pick)]
+    gidx = [gk[ix] for gk, ix in zip(g, pick)]
+    es.es_replay(plan, seeds, coeffs, counts)
+    torch.cuda.synchronize()
+
+    def values(x):
+        return bf16_values(x) if dtype == "bf16" else np.asarray(x, dtype=np.float64)
+
+    tol = [0.0] * len(segs)
+    peak = [np.abs(values(x)) for x in state]
+    for a, b in zip(starts, ends):
+        for k in range(len(segs)):
+            state[k] = oracle.update(state[k], gidx[k], seeds[a:b], coeffs[a:b], dtype)
+            tol[k] = tol[k] + noise_abs_tol(
+                [oracle.noise_at(int(sd), gidx[k]) for sd in seeds[a:b]], coeffs[a:b])
+            peak[k] = np.maximum(peak[k], np.abs(values(state[k])))
+    # Each generation rounds once on both sides: the GPU from an fp32 sum, the
+    # oracle from a double one. Where the exact value lies within the fp32 sum's
+    # error of a rounding tie, the two round to neighbouring values one unit in
+    # the last place apart, and later generations carry that absolute
+    # difference even after |theta| has shrunk. So the replay is held to the
+    # step's unit: two units in the last place of the largest |theta| the
+    # element took along the oracle's trajectory (bf16), or the per-call
+    # relative bound 1e-5 of that magnitude (fp32), plus the carried noise
+    # tolerance; and for bf16 at most 0.1 % of the elements may differ by more
+    # than one such unit.
+    for k in range(len(segs)):
+        got = values(host_values(tensors[k])[pick[k]])
+        want = values(state[k])
+        err = np.abs(got - want)
+        if dtype == "bf16":
+            unit = 2.0 ** (np.floor(np.log2(np.maximum(peak[k], 2.0**-126))) - 7)
+            bad = err > 2 * unit + tol[k]
+            far = err > unit + tol[k]
+            assert np.count_nonzero(far) <= max(1, got.size // 1000), f"replay seg {k}"
+        else:
+            bad = err > 1e-5 * peak[k] + tol[k]
+        assert not np.any(bad), (f"replay seg {k}: {np.count_nonzero(bad)} elements; first "
+                                 f"got {got[bad][:3]} want {want[bad][:3]}")
+    plan.close()
+
+
+@pytest.mark.parametrize("dtype", ["bf16", "f32"])
+def test_antithetic_flip_matches_oracle(es, oracle, dtype):
+    # The flip of an antithetic pair, es_restore_perturb(s, sigma, s, -sigma),
+    # takes theta + sigma eps_s to theta - sigma eps_s in one pass with the
+    # noise generated once: restore, then perturb with -sigma (§3), each
+    # rounded to storage. Against the oracle's two steps from the GPU's input,
+    # over several flips and seeds, on ragged 64-bit layouts.
+    tensors = make_params(dtype, RAGGED, seed=42)
+    plan, segs = build_plan(es, tensors, _sparse64(len(RAGGED)))
+    g = indices(segs)
+    for seed, sigma in ((31, 5e-2), (2**41 + 9, 1e-3), (2**63 + 5, 2.5e-4)):
+        es.es_perturb(plan, seed, sigma)
+        torch.cuda.synchronize()
+        before = [host_values(t) for t in tensors]
+        es.es_restore_perturb(plan, seed, sigma, seed, -sigma)
+        torch.cuda.synchronize()
+        # Two roundings (restore, then perturb), and the intermediate is not
+        # observable: where the GPU and the oracle round the intermediate to
+        # neighbouring values, that one-ulp difference at the intermediate's
+        # magnitude is carried into the result, and the second rounding can add
+        # one ulp at the result's. bf16 is held to that sum (plus the carried
+        # noise tolerance), with at most 0.1 % of the elements beyond one ulp of
+        # the larger magnitude; fp32 to the per-call relative bound of it. The
+        # fused flip is also bit-identical to the two separate calls, each
+        # checked one step at a time elsewhere.
+        for k in range(len(tensors)):
+            eps = oracle.noise_at(seed, g[k])
+            mid = oracle.restore(before[k], g[k], seed, sigma, dtype)
+            want = oracle.perturb(mid, g[k], seed, -sigma, dtype)
+            got = host_values(tensors[k])
+            tol = noise_abs_tol([eps, eps], [sigma, sigma])
+            if dtype == "bf16":
+                g_v, w_v, m_v = bf16_values(got), bf16_values(want), bf16_values(mid)
+
+                def ulp(x):
+                    return 2.0 ** (np.floor(np.log2(np.maximum(np.abs(x), 2.0**-126))) - 7)
+
+                err = np.abs(g_v - w_v)
+                bound = ulp(m_v) + ulp(w_v) + tol
+                assert np.all(err <= bound), f"flip seed {seed} seg {k}"
+                far = err > np.maximum(ulp(m_v), ulp(w_v)) + tol
+                assert np.count_nonzero(far) <= max(1, got.size // 1000), f"flip seed {seed} seg {k}"
+            else:
+                m_v = np.abs(np.asarray(mid, dtype=np.float64))
+                err = np.abs(got.astype(np.float64) - np.asarray(want, dtype=np.float64))
+                assert np.all(err <= 1e-5 * np.maximum(m_v, np.abs(want)) + tol), \
+                    f"flip seed {seed} seg {k}"
+        es.es_restore(plan, seed, -sigma)
+    plan.close()
 
 
 def test_replay_argument_errors(es):
