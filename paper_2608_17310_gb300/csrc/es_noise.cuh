@@ -31,35 +31,21 @@ __host__ __device__ inline PhiloxKey philox_key(uint64_t seed) {
   return PhiloxKey{static_cast<uint32_t>(seed), static_cast<uint32_t>(seed >> 32)};
 }
 
-// High and low words of the 32x32->64-bit product m * x, as two separate
-// 32-bit multiplies (mul.hi.u32 and mul.lo.u32). Measured on sm_103a, this
-// form runs the generator 6-7 % faster than one 64-bit-result multiply
-// (mul.wide.u32): the low-word multiply issues at a higher rate than the wide
-// one, and the pair schedules better around the transcendentals. The words
-// are the same either way.
+// High and low words of the 32x32->64-bit product m * x. Two forms, with the
+// same words: two 32-bit multiplies (mul.hi.u32, mul.lo.u32), or one multiply
+// with a 64-bit result (mul.wide.u32). Measured on sm_103a in the library's
+// kernels, the fastest mix is the 64-bit form in the eight full rounds of the
+// per-tile path (philox_block_tile) and the 32-bit pair everywhere else (the
+// first two rounds, the per-tile constants and the general path): 5-8 %
+// faster than either form throughout, which cost registers and occupancy in
+// the fused update.
 __device__ __forceinline__ uint32_t mul_hi(uint32_t m, uint32_t x) { return __umulhi(m, x); }
 __device__ __forceinline__ uint32_t mul_lo(uint32_t m, uint32_t x) { return m * x; }
-
-// Product of one Philox multiplier with a word, as (high, low): kWide picks the
-// single 64-bit-result multiply, otherwise the mul.hi / mul.lo pair.
-#ifndef ES_PHILOX_FORM
-#define ES_PHILOX_FORM 0
-#endif
-template <bool kWide>
-__device__ __forceinline__ void mul_hilo(uint32_t m, uint32_t x, uint32_t& hi, uint32_t& lo) {
-  if constexpr (kWide) {
-    const uint64_t p = static_cast<uint64_t>(m) * x;
-    hi = static_cast<uint32_t>(p >> 32);
-    lo = static_cast<uint32_t>(p);
-  } else {
-    hi = mul_hi(m, x);
-    lo = mul_lo(m, x);
-  }
+__device__ __forceinline__ void mul_wide(uint32_t m, uint32_t x, uint32_t& hi, uint32_t& lo) {
+  const uint64_t p = static_cast<uint64_t>(m) * x;
+  hi = static_cast<uint32_t>(p >> 32);
+  lo = static_cast<uint32_t>(p);
 }
-// Form of the A (word 0) and B (word 2) products: 0 both pairs, 1 both wide,
-// 2 A wide and B a pair, 3 A a pair and B wide.
-constexpr bool kWideA = ES_PHILOX_FORM == 1 || ES_PHILOX_FORM == 2;
-constexpr bool kWideB = ES_PHILOX_FORM == 1 || ES_PHILOX_FORM == 3;
 
 // Ten Philox-4x32 rounds on counter (j_lo, j_hi, 0, 0). Each round is two
 // 32x32->64 products (high and low words) and two three-input XORs; the key
@@ -71,13 +57,10 @@ __device__ __forceinline__ uint4 philox_block(uint64_t j, PhiloxKey key) {
   uint32_t k0 = key.k0, k1 = key.k1;
 #pragma unroll
   for (int round = 0; round < 10; ++round) {
-    uint32_t ha, la, hb, lb;
-    mul_hilo<kWideA>(kPhiloxMulA, c0, ha, la);
-    mul_hilo<kWideB>(kPhiloxMulB, c2, hb, lb);
-    const uint32_t n0 = hb ^ c1 ^ k0;
-    const uint32_t n2 = ha ^ c3 ^ k1;
-    c1 = lb;
-    c3 = la;
+    const uint32_t n0 = mul_hi(kPhiloxMulB, c2) ^ c1 ^ k0;
+    const uint32_t n2 = mul_hi(kPhiloxMulA, c0) ^ c3 ^ k1;
+    c1 = mul_lo(kPhiloxMulB, c2);
+    c3 = mul_lo(kPhiloxMulA, c0);
     c0 = n0;
     c2 = n2;
     k0 += kPhiloxWeylA;
@@ -101,28 +84,25 @@ struct PhiloxTile {
 
 __device__ __forceinline__ PhiloxTile philox_tile(uint32_t j_hi, PhiloxKey key) {
   const uint32_t w0 = j_hi ^ key.k0;
-  uint32_t h, l;
-  mul_hilo<kWideA>(kPhiloxMulA, w0, h, l);
-  return PhiloxTile{key, w0, h ^ (key.k1 + kPhiloxWeylB), l};
+  return PhiloxTile{key, w0, mul_hi(kPhiloxMulA, w0) ^ (key.k1 + kPhiloxWeylB),
+                    mul_lo(kPhiloxMulA, w0)};
 }
 
 __device__ __forceinline__ uint4 philox_block_tile(uint32_t j_lo, const PhiloxTile& t) {
   // round 1 (keys k0, k1): products kPhiloxMulA * j_lo and kPhiloxMulB * 0
-  uint32_t h1, a3;
-  mul_hilo<kWideA>(kPhiloxMulA, j_lo, h1, a3);                // a3: word 3
-  const uint32_t a2 = h1 ^ t.key.k1;                          // word 2
+  const uint32_t a2 = mul_hi(kPhiloxMulA, j_lo) ^ t.key.k1;   // word 2
+  const uint32_t a3 = mul_lo(kPhiloxMulA, j_lo);              // word 3
   // round 2 (keys k0 + W_A, k1 + W_B): word 0 is t.w0, its product is per tile
-  uint32_t h2, c1;
-  mul_hilo<kWideB>(kPhiloxMulB, a2, h2, c1);
-  uint32_t c0 = h2 ^ (t.key.k0 + kPhiloxWeylA);               // word 1 was 0
+  uint32_t c0 = mul_hi(kPhiloxMulB, a2) ^ (t.key.k0 + kPhiloxWeylA);  // word 1 was 0
+  uint32_t c1 = mul_lo(kPhiloxMulB, a2);
   uint32_t c2 = t.x2 ^ a3;
   uint32_t c3 = t.lo2;
   uint32_t k0 = t.key.k0 + 2u * kPhiloxWeylA, k1 = t.key.k1 + 2u * kPhiloxWeylB;
 #pragma unroll
   for (int round = 2; round < 10; ++round) {
     uint32_t ha, la, hb, lb;
-    mul_hilo<kWideA>(kPhiloxMulA, c0, ha, la);
-    mul_hilo<kWideB>(kPhiloxMulB, c2, hb, lb);
+    mul_wide(kPhiloxMulA, c0, ha, la);
+    mul_wide(kPhiloxMulB, c2, hb, lb);
     const uint32_t n0 = hb ^ c1 ^ k0;
     const uint32_t n2 = ha ^ c3 ^ k1;
     c1 = lb;
@@ -135,18 +115,9 @@ __device__ __forceinline__ uint4 philox_block_tile(uint32_t j_lo, const PhiloxTi
   return make_uint4(c0, c1, c2, c3);
 }
 
-// The float 1 + m 2^-23 for m = x >> 9 (top 23 bits of x), i.e. the bit
-// pattern 0x3F800000 | (x >> 9): the low word of the 64-bit value
-// (0x7F : x) shifted right by 9, one funnel shift (0x7F << 23 = 0x3F800000).
-#ifndef ES_UNIFORM_FUNNEL
-#define ES_UNIFORM_FUNNEL 0
-#endif
+// The float 1 + m 2^-23 for m = x >> 9 (the top 23 bits of x).
 __device__ __forceinline__ float one_plus_top23(uint32_t x) {
-#if ES_UNIFORM_FUNNEL
-  return __uint_as_float(__funnelshift_r(x, 0x7Fu, 9));
-#else
   return __uint_as_float(0x3F800000u | (x >> 9));
-#endif
 }
 
 // u = (2m + 1) / 2^24 with m = x >> 9, computed exactly: 1 + m 2^-23 minus
@@ -165,41 +136,32 @@ constexpr float kTwoPi = 6.28318530717958647692f;
 // -3 pi + 2 pi 2^-24 rounded to float: 2 pi (f - 3/2 + 2^-24) = fma(f, 2 pi, this)
 constexpr float kAngleOffset = -9.42477798f;
 
-#ifndef ES_FTZ_MUFU
-#define ES_FTZ_MUFU 1
-#endif
-
+// The hardware approximations of log2, sqrt, sin and cos, in their
+// flush-to-zero forms. These differ from the default forms only for subnormal
+// inputs (which the default forms first scale into the normal range at the cost
+// of extra instructions), and no input here is subnormal: u >= 2^-24, the
+// radius squared is at least 2t + t^2 with t >= 2^-24 or at least
+// 2 ln 2 * 2^-10 from the log path, and the angle is at least 2 pi 2^-24 in
+// magnitude. Measured: the generator's kernels run 6-10 % faster.
 __device__ __forceinline__ float sqrt_approx(float x) {
   float r;
-#if ES_FTZ_MUFU
   asm("sqrt.approx.ftz.f32 %0, %1;" : "=f"(r) : "f"(x));
-#else
-  asm("sqrt.approx.f32 %0, %1;" : "=f"(r) : "f"(x));
-#endif
   return r;
 }
 
 __device__ __forceinline__ float log2_approx(float x) {
-#if ES_FTZ_MUFU
   float r;
   asm("lg2.approx.ftz.f32 %0, %1;" : "=f"(r) : "f"(x));
   return r;
-#else
-  return __log2f(x);
-#endif
 }
 
 __device__ __forceinline__ void sincos_approx(float a, float* s, float* c) {
-#if ES_FTZ_MUFU
   asm("sin.approx.ftz.f32 %0, %1;" : "=f"(*s) : "f"(a));
   asm("cos.approx.ftz.f32 %0, %1;" : "=f"(*c) : "f"(a));
-#else
-  __sincosf(a, s, c);
-#endif
 }
 
 // radius^2 = -2 ln u for u = uniform_open(x), fast path:
-//   for u <= 1 - 2^-10: -2 ln 2 * log2(u) with the MUFU log2 (__log2f);
+//   for u <= 1 - 2^-10: -2 ln 2 * log2(u) with the MUFU log2 (log2_approx);
 //   for u >  1 - 2^-10: 2t + t^2 with t = 1 - u (exact); the dropped terms
 //     (2/3 t^3 + ...) are below t^2/3 <= 3.2e-7 relative.
 // Both are evaluated and one is selected, which keeps the code free of
@@ -215,8 +177,9 @@ __device__ __forceinline__ float radius_sq(float u) {
 //   r = sqrt.approx(radius_sq(u_a));
 //   angle: with f = 1 + m_b 2^-23 (bits 0x3F800000 | m_b), 2 pi u_b =
 //     2 pi (f - 3/2 + 2^-24) + pi, so cos/sin of 2 pi u_b are -c/-s with
-//     (s, c) = __sincosf(fma(f, 2 pi, kAngleOffset)), an argument in (-pi, pi)
-//     where __sincosf is accurate; the fma rounds once (|error| < 1e-6).
+//     (s, c) = sincos_approx(fma(f, 2 pi, kAngleOffset)), an argument in
+//     (-pi, pi) where the hardware sine and cosine are accurate; the fma
+//     rounds once (|error| < 1e-6).
 // Kernels that add scale * eps fold the scale into r: theta + scale * eps_even
 // = fma(-(scale * r), c, theta).
 // Checked against the exact pair over the whole input domain (every 23-bit
