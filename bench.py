@@ -344,6 +344,8 @@ IMUL_PER_CLK_SM = 64
 # per clock per SM): 2 per Gaussian.
 MUFU_PER_GAUSS = 2
 MUFU_PER_CLK_SM = 16
+# Three-input XORs of those rounds (lop3): 19 per block of 4 Gaussians.
+LOP3_PER_GAUSS = 19 / 4
 
 
 # The device code of the kernels whose DRAM traffic is recorded.
@@ -466,7 +468,7 @@ def run_ours(args, rank, world, dist):
     per_step_ms = ms_max / args.steps
     value = world * P * n * args.steps / (ms_max / 1e3)
 
-    imul_peak, gauss_peak, shared_peak, sms, sm_max_mhz, hbm_gbs, peak_src, ceilings = \
+    imul_peak, gauss_peak, measured_peak, sms, sm_max_mhz, hbm_gbs, peak_src, ceilings = \
         alu_peaks(torch, dev_index)
     bytes_per_launch = 2 * esize * P
     kernels = {}
@@ -479,7 +481,7 @@ def run_ours(args, rank, world, dist):
         kernels[name] = {"kernel": KERNEL_NAME[name], "launches": timers.count(name),
                          "mean_ms": mean, "share": timers.total_ms(name) / ms,
                          "gbs": gbs, "gauss_per_s": gps, "hbm_frac": hbm_frac,
-                         "alu_frac": alu_frac, "imul_mufu_frac": gps / shared_peak,
+                         "alu_frac": alu_frac, "measured_alu_frac": gps / measured_peak,
                          "bound": "alu" if alu_frac > hbm_frac else "hbm"}
     dom = max(kernels, key=lambda k: kernels[k]["share"])
     d = kernels[dom]
@@ -495,11 +497,13 @@ def run_ours(args, rank, world, dist):
                 "traffic": traffic,
                 "peak_source": f"{sms} SMs x {IMUL_PER_CLK_SM} 32-bit integer multiplies/clk x "
                                f"{sm_max_mhz:.0f} MHz; {IMUL_PER_GAUSS} multiplies per Gaussian"}
-    roof["imul_mufu_bound"] = {
-        "gauss_per_s": shared_peak, "frac": d["gauss_per_s"] / shared_peak,
-        "source": "measured in this run: register-only probe of mad.wide.u32 and MUFU in the "
-                  "generator's ratio (9:4) in one thread, 4 CTAs per SM, scaled to the "
-                  "maximum SM clock (bench.py --pipe-peaks has every probe)"}
+    roof["measured_alu_bound"] = {
+        "gauss_per_s": measured_peak, "frac": d["gauss_per_s"] / measured_peak,
+        "binding_pipe": ceilings["alu"]["binding_pipe"],
+        "source": "measured in this run: the method's mandated ALU work per Gaussian (4.5 "
+                  "mad.wide.u32, 4.75 lop3, 2 MUFU) over each pipe's rate in register-only "
+                  "probes at 4 CTAs per SM, the slowest pipe binding, scaled to the maximum SM "
+                  "clock (bench.py --pipe-peaks has every probe)"}
     roof["measured_ceilings"] = ceilings
     roof["pipe_occupancy"] = pipe_occupancy(dom)
     roof.update({"kernel": d["kernel"], "hbm_frac": d["hbm_frac"], "alu_frac": d["alu_frac"],
@@ -576,30 +580,32 @@ def measured_ceilings(res, sms, sm_max_mhz):
     """ALU ceilings of the generator from probe results (`res`: name -> run_probe
     dict), in Gaussians/s at the maximum SM clock:
       imad_wide      the integer-multiply pipe alone: mad.wide.u32 rate / 4.5;
+      lop3           the three-input XOR alone: lop3 rate / 4.75;
       mufu           the MUFU pipe alone: its rate / 2;
-      imad_mufu_mix  both in the generator's ratio (9 mad.wide : 4 MUFU) in one
-                     thread: the shared ceiling of this formulation;
+      alu            the bound of the method's mandated ALU work with these
+                     measured pipe peaks: t_ALU per Gaussian = the maximum over
+                     the three pipes of mandated ops / measured rate;
+      imad_mufu_mix  mad.wide and MUFU in the generator's ratio (9 : 4) in one
+                     thread;
       generator      the library's full generator (Philox + Box-Muller) in
                      registers, no memory traffic."""
     hz = sms * sm_max_mhz * 1e6
     out = {}
-    if "imad_wide" in res:
-        r = res["imad_wide"]["ops_per_clk_sm"]
-        out["imad_wide"] = {"ops_per_clk_sm": r, "imul32_per_clk_sm": 2 * r,
-                            "gauss_per_s": r / WIDE_PER_GAUSS * hz}
-    if "mufu" in res:
-        r = res["mufu"]["ops_per_clk_sm"]
-        out["mufu"] = {"ops_per_clk_sm": r, "gauss_per_s": r / MUFU_PER_GAUSS * hz}
+    per_pipe = {}
+    for name, per_g in (("imad_wide", WIDE_PER_GAUSS), ("lop3", LOP3_PER_GAUSS),
+                        ("mufu", MUFU_PER_GAUSS)):
+        if name in res:
+            r = res[name]["ops_per_clk_sm"]
+            out[name] = {"ops_per_clk_sm": r, "per_gaussian": per_g, "gauss_per_s": r / per_g * hz}
+            per_pipe[name] = r / per_g * hz
+    if "imad_wide" in out:
+        out["imad_wide"]["imul32_per_clk_sm"] = 2 * out["imad_wide"]["ops_per_clk_sm"]
+    if per_pipe:
+        pipe = min(per_pipe, key=per_pipe.get)
+        out["alu"] = {"gauss_per_s": per_pipe[pipe], "binding_pipe": pipe}
     if "mix_imad_wide_mufu_9_4" in res:
         r = res["mix_imad_wide_mufu_9_4"]["ops_per_clk_sm"]
         out["imad_mufu_mix"] = {"wide_per_clk_sm": r, "gauss_per_s": r / WIDE_PER_GAUSS * hz}
-        if "imad_wide" in out and "mufu" in out:
-            a, m = out["imad_wide"]["ops_per_clk_sm"], out["mufu"]["ops_per_clk_sm"]
-            additive = 1.0 / (WIDE_PER_GAUSS / a + MUFU_PER_GAUSS / m)
-            overlapped = min(a / WIDE_PER_GAUSS, m / MUFU_PER_GAUSS)
-            out["imad_mufu_mix"].update({
-                "gauss_per_s_if_additive": additive * hz,
-                "gauss_per_s_if_overlapped": overlapped * hz})
     if "mix_imad_hi_lo_1_1" in res:
         r = res["mix_imad_hi_lo_1_1"]["ops_per_clk_sm"]
         out["imad_hi_lo"] = {"pairs_per_clk_sm": r, "imul32_per_clk_sm": 2 * r,
@@ -619,33 +625,35 @@ def measured_ceilings(res, sms, sm_max_mhz):
     return out
 
 
-CEILING_PROBES = ("imad_wide", "mufu", "mix_imad_wide_mufu_9_4", "mix_imad_hi_lo_1_1",
+CEILING_PROBES = ("imad_wide", "lop3", "mufu", "mix_imad_wide_mufu_9_4", "mix_imad_hi_lo_1_1",
                   "mix_imad_hi_lo_mufu_9_4", "generator")
 
 
 def alu_peaks(torch, dev_index, probes=True):
     """(imul32/s at the nominal integer-multiply rate, Gaussians/s at that
-    roofline, Gaussians/s at the measured shared IMUL+MUFU ceiling, SM count,
-    max SM MHz, HBM GB/s, peak source, measured ceilings).
+    roofline, Gaussians/s at the measured ALU bound, SM count, max SM MHz, HBM
+    GB/s, peak source, measured ceilings).
 
     The roofline is the nominal one: 64 32-bit multiplies per clock per SM x
-    SMs x the maximum SM clock, 9 multiplies per Gaussian. The shared ceiling is
-    measured live by the register-only probes (the generator's mix of
-    mad.wide.u32 and MUFU in one thread); without probes it is None."""
+    SMs x the maximum SM clock, 9 multiplies per Gaussian. The measured ALU
+    bound takes the same mandated work against the pipe peaks that the
+    register-only probes measure live (mad.wide.u32, lop3, MUFU; the slowest
+    pipe binds); without probes it is None."""
     hbm_gbs, sm_max_mhz, peak_src = peaks()
     sms = torch.cuda.get_device_properties(dev_index).multi_processor_count
     imul_peak = sms * IMUL_PER_CLK_SM * sm_max_mhz * 1e6
     ceilings = {}
-    shared_peak = None
+    measured_peak = None
     if probes:
         L = probe_lib()
         res = {name: run_probe(L, name, 4, 10.0) for name in CEILING_PROBES}
         ceilings = measured_ceilings(res, sms, sm_max_mhz)
         ceilings["source"] = ("bench.py probes (csrc/es_probes.cu): register-only loops, 4 CTAs "
-                              "of 256 threads per SM, rates in SM cycles scaled to the maximum "
+                              "of 256 threads per SM, each SM timed on its own clock from its "
+                              "first CTA's start to its last CTA's end, scaled to the maximum "
                               "SM clock")
-        shared_peak = ceilings["imad_mufu_mix"]["gauss_per_s"]
-    return (imul_peak, imul_peak / IMUL_PER_GAUSS, shared_peak, sms, sm_max_mhz, hbm_gbs,
+        measured_peak = ceilings["alu"]["gauss_per_s"]
+    return (imul_peak, imul_peak / IMUL_PER_GAUSS, measured_peak, sms, sm_max_mhz, hbm_gbs,
             peak_src, ceilings)
 
 
@@ -699,7 +707,7 @@ def run_sweep(args, rank, world, dist):
     P = plan.numel
     stream = torch.cuda.current_stream()
     s_handle = stream.cuda_stream
-    imul_peak, gauss_peak, shared_peak, sms, sm_max_mhz, hbm_gbs, peak_src, _ = \
+    imul_peak, gauss_peak, measured_peak, sms, sm_max_mhz, hbm_gbs, peak_src, _ = \
         alu_peaks(torch, dev_index)
     bytes_per_launch = 2 * esize * P
     pops = [int(x) for x in args.populations.split(",") if x.strip()]
@@ -731,14 +739,15 @@ def run_sweep(args, rank, world, dist):
             gps = n * P / (ms / 1e3)
             t_hbm = bytes_per_launch / (hbm_gbs * 1e9) * 1e3
             t_imul = n * P / gauss_peak * 1e3
-            t_shared = n * P / shared_peak * 1e3
+            t_measured = n * P / measured_peak * 1e3
             points.append({
                 "population": n, "mean_ms": ms, "gbs": gbs, "gauss_per_s": gps,
                 "hbm_frac": gbs / hbm_gbs, "alu_frac": gps / gauss_peak,
-                "imul_mufu_frac": gps / shared_peak,
+                "measured_alu_frac": gps / measured_peak,
                 "bound": "alu" if t_imul > t_hbm else "hbm",
                 "roofline_frac": max(t_hbm, t_imul) / ms,
-                "t_hbm_ms": t_hbm, "t_imul_ms": t_imul, "t_imul_mufu_ms": t_shared})
+                "measured_roofline_frac": max(t_hbm, t_measured) / ms,
+                "t_hbm_ms": t_hbm, "t_imul_ms": t_imul, "t_alu_measured_ms": t_measured})
     plan.close()
     out = {"mode": "sweep", "metric": "es_update param*seed/s per population size",
            "unit": UNIT, "n_gpus": 1, "steps": args.steps, "warmup": args.warmup,
@@ -748,7 +757,8 @@ def run_sweep(args, rank, world, dist):
                           rewards="N(0,1) used as the normalised rewards; paper-scale coefficients"),
            "peaks": {"hbm_gbs": hbm_gbs, "hbm_source": peak_src,
                      "imul32_per_s": imul_peak, "gauss_per_s_imul": gauss_peak,
-                     "gauss_per_s_imul_mufu": shared_peak, "sms": sms, "sm_max_mhz": sm_max_mhz},
+                     "gauss_per_s_alu_measured": measured_peak, "sms": sms,
+                     "sm_max_mhz": sm_max_mhz},
            "bytes_per_launch": bytes_per_launch, "points": points,
            "gpu_launches": launches, "clocks": clk.summary()}
     if rank == 0:
@@ -769,11 +779,11 @@ def _timed(torch, stream, fn, reps):
 
 
 def _rates(P, gaussians_per_param, bytes_total, ms, peaks_):
-    imul_peak, gauss_peak, shared_peak, _, _, hbm_gbs, _, _ = peaks_
+    imul_peak, gauss_peak, measured_peak, _, _, hbm_gbs, _, _ = peaks_
     gps = gaussians_per_param * P / (ms / 1e3)
     gbs = bytes_total / (ms / 1e3) / 1e9
     return {"ms": ms, "gauss_per_s": gps, "gbs": gbs, "hbm_frac": gbs / hbm_gbs,
-            "alu_frac": gps / gauss_peak, "imul_mufu_frac": gps / shared_peak}
+            "alu_frac": gps / gauss_peak, "measured_alu_frac": gps / measured_peak}
 
 
 def run_replay(args, rank, world, dist):

@@ -17,28 +17,42 @@ constexpr int kBlockThreads = 256;
 // straddle segments.
 constexpr int kVecsPerThread = 4;
 
-// Per kernel kind (one-seed pass, two-seed pass, update): how many of its
-// tile vectors a thread processes at once (the group; each vector is
-// vec_elems / 4 independent Philox chains), and the resident CTAs per SM asked
-// of the compiler (a register cap; 1 leaves registers to the compiler). A
-// smaller group needs fewer registers, so more warps fit on an SM.
+// Per kernel kind (one-seed pass, two-seed pass, update): how many 16-byte
+// vectors of its tile a thread processes at once (the group; each bf16 vector
+// is two independent Philox chains per seed), the resident CTAs per SM asked
+// of the compiler (a register cap), and the instruction form of the noise step
+// (0 scalar FP32, 1 scalar transform with packed FMAs, 2 packed; the values
+// are bit-identical). Measured on sm_103a over the 4B-shaped set: one vector
+// at a time at 3 CTAs per SM is fastest for every kernel; more CTAs per SM,
+// larger groups or a second seed in flight gain nothing, since the generator
+// is bound by the FMA-heavy pipe (its integer products and packed FP32), not
+// by latency.
 #ifndef ES_AXPY1_GROUP
-#define ES_AXPY1_GROUP 4
+#define ES_AXPY1_GROUP 1
 #endif
 #ifndef ES_AXPY1_MIN_BLOCKS
-#define ES_AXPY1_MIN_BLOCKS 1
+#define ES_AXPY1_MIN_BLOCKS 3
+#endif
+#ifndef ES_AXPY1_FORM
+#define ES_AXPY1_FORM 2
 #endif
 #ifndef ES_AXPY2_GROUP
-#define ES_AXPY2_GROUP 4
+#define ES_AXPY2_GROUP 1
 #endif
 #ifndef ES_AXPY2_MIN_BLOCKS
-#define ES_AXPY2_MIN_BLOCKS 1
+#define ES_AXPY2_MIN_BLOCKS 3
+#endif
+#ifndef ES_AXPY2_FORM
+#define ES_AXPY2_FORM 2
 #endif
 #ifndef ES_UPDATE_GROUP
-#define ES_UPDATE_GROUP 4
+#define ES_UPDATE_GROUP 1
 #endif
 #ifndef ES_UPDATE_MIN_BLOCKS
-#define ES_UPDATE_MIN_BLOCKS 1
+#define ES_UPDATE_MIN_BLOCKS 3
+#endif
+#ifndef ES_UPDATE_FORM
+#define ES_UPDATE_FORM 1
 #endif
 // Seeds of the update's seed loop issued together (independent generator
 // work per element across seeds; the accumulation stays in ascending order).

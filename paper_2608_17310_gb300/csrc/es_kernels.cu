@@ -28,8 +28,6 @@ struct Bf16Io {
   static constexpr int kVec = 8;
   static constexpr bool kScaled = false;
   using Scalar = uint16_t;
-  __device__ static float to_f32(uint16_t h) { return __uint_as_float(static_cast<uint32_t>(h) << 16); }
-  __device__ static uint16_t from_f32(float f) { return __bfloat16_as_ushort(__float2bfloat16_rn(f)); }
   __device__ static uint32_t pack2(float lo, float hi) {
     __nv_bfloat162 h = __floats2bfloat162_rn(lo, hi);  // one cvt.rn.bf16x2.f32
     return *reinterpret_cast<uint32_t*>(&h);
@@ -73,8 +71,6 @@ struct F32Io {
   static constexpr int kVec = 4;
   static constexpr bool kScaled = false;
   using Scalar = float;
-  __device__ static float to_f32(float f) { return f; }
-  __device__ static float from_f32(float f) { return f; }
   __device__ static void unpack(const uint4& v, float (&f)[4]) {
     f[0] = __uint_as_float(v.x); f[1] = __uint_as_float(v.y);
     f[2] = __uint_as_float(v.z); f[3] = __uint_as_float(v.w);
@@ -118,13 +114,6 @@ struct Fp8Io {
     return static_cast<uint32_t>(__nv_cvt_float2_to_fp8x2(make_float2(lo, hi), __NV_SATFINITE,
                                                           __NV_E4M3));
   }
-  __device__ static float to_f32(uint8_t c) {
-    return __half2float(__half(__nv_cvt_fp8_to_halfraw(static_cast<__nv_fp8_storage_t>(c),
-                                                       __NV_E4M3)));
-  }
-  __device__ static uint8_t from_f32(float f) {
-    return static_cast<uint8_t>(__nv_cvt_float_to_fp8(f, __NV_SATFINITE, __NV_E4M3));
-  }
   __device__ static void unpack(const uint4& v, float (&f)[16]) {
     const uint32_t w[4] = {v.x, v.y, v.z, v.w};
 #pragma unroll
@@ -165,11 +154,12 @@ struct Fp8Io {
   }
 };
 
-// Vectors a thread processes at once for a kernel kind's group g: FP8 vectors
-// hold twice the elements of bf16 ones, so they go half as many at a time.
+// Vectors a thread processes at once for a kernel kind's group g (g bf16
+// vectors of 8 elements): the same number of elements, hence of Philox
+// chains, for every storage type, within the kVecsPerThread vectors of a tile.
 template <class Io>
 __host__ __device__ constexpr int group_for(int g) {
-  return Io::kVec > 8 ? (g > 1 ? g / 2 : 1) : g;
+  return Io::kVec > 8 ? (g > 1 ? g / 2 : 1) : Io::kVec < 8 ? (2 * g < kVecsPerThread ? 2 * g : kVecsPerThread) : g;
 }
 
 // theta + acc in storage units: acc is in parameter units, so a scaled
@@ -182,10 +172,21 @@ __device__ __forceinline__ float add_acc(float theta, float acc, float inv_scale
 
 // Philox words of block j for one seed. TileGen serves the blocks of a tile
 // that share the high counter word (per-tile constants, see philox_tile);
-// AnyGen serves any block. Both give the same words.
+// SchedGen does the same with the round keys read from a precomputed schedule
+// (kernel parameters or registers loaded from shared memory); AnyGen serves
+// any block. All give the same words.
 struct TileGen {
   PhiloxTile t;
   __device__ uint4 block(uint64_t j) const { return philox_block_tile(static_cast<uint32_t>(j), t); }
+};
+template <class Keys>
+struct SchedGen {
+  TileConst t;
+  uint32_t rk1, rk2;  // round 0's k1, round 1's k0
+  Keys rk;            // rounds 2..9: rk[2r - 4], rk[2r - 3]
+  __device__ uint4 block(uint64_t j) const {
+    return philox_block_rk(static_cast<uint32_t>(j), t, rk1, rk2, rk);
+  }
 };
 struct AnyGen {
   PhiloxKey key;
@@ -198,6 +199,14 @@ __device__ __forceinline__ auto make_gen(PhiloxKey key, uint32_t j_hi) {
   else return AnyGen{key};
 }
 
+// Generator of one seed whose schedule is a kernel parameter.
+template <bool kUniformHi>
+__device__ __forceinline__ auto sched_gen(const PhiloxSched& s, uint32_t j_hi) {
+  if constexpr (kUniformHi)
+    return SchedGen<const uint32_t*>{tile_const(j_hi, s.rk[0], s.rk[3]), s.rk[1], s.rk[2], s.rk + 4};
+  else return AnyGen{PhiloxKey{s.rk[0], s.rk[1]}};
+}
+
 // How each Philox block becomes theta updates. The forms give bit-identical
 // values: a packed two-wide FP32 instruction rounds each half exactly like the
 // scalar one. They differ only in instruction mix, which moves work between the
@@ -206,6 +215,9 @@ __device__ __forceinline__ auto make_gen(PhiloxKey key, uint32_t j_hi) {
 //   kPackedFma  scalar transform, packed FMAs into theta or the accumulator;
 //   kPacked     packed transform (polar2) and packed FMAs.
 enum class NoiseForm { kScalar, kPackedFma, kPacked };
+constexpr NoiseForm kAxpy1Form = static_cast<NoiseForm>(ES_AXPY1_FORM);
+constexpr NoiseForm kAxpy2Form = static_cast<NoiseForm>(ES_AXPY2_FORM);
+constexpr NoiseForm kUpdateForm = static_cast<NoiseForm>(ES_UPDATE_FORM);
 
 // f[k] += scale * eps[g0 + k] for the V elements from global index g0
 // (g0 % 4 == 0), with scale folded into each pair's radius.
@@ -283,76 +295,112 @@ __device__ __forceinline__ bool uniform_hi(uint64_t index_base, uint64_t t0, uin
   return ((index_base + t0) >> 34) == (last >> 34);
 }
 
-// Location of one tile: its segment's storage and the tile's first element.
+// Location of one tile: its segment's storage, the tile's first element and,
+// for a scaled storage type, 1 / the segment's scale.
 template <class Io>
 struct TileRef {
   typename Io::Scalar* base;
   uint64_t numel;
   uint64_t index_base;
   uint64_t t0;
+  float inv;
 };
 
 template <class Io>
-__device__ __forceinline__ TileRef<Io> tile_ref(const SegDesc* __restrict__ segs, int& seg,
-                                                uint64_t tile, uint64_t tile_elems) {
+__device__ __forceinline__ TileRef<Io> tile_ref(const SegDesc* __restrict__ segs,
+                                                const float* __restrict__ inv_scale, int& seg,
+                                                uint64_t tile) {
+  constexpr uint64_t kTile = static_cast<uint64_t>(kBlockThreads) * kVecsPerThread * Io::kVec;
   const SegDesc* d = find_segment(segs, seg, tile);
   return TileRef<Io>{static_cast<typename Io::Scalar*>(d->data), d->numel, d->index_base,
-                     (tile - d->tile_begin) * tile_elems};
+                     (tile - d->tile_begin) * kTile, Io::kScaled ? inv_scale[seg] : 1.0f};
 }
 
-// One tile of the perturb/restore pass (kTwo: fused restore + perturb; kSame:
-// both steps use one seed, whose noise is generated once). Each thread takes
-// its kVecsPerThread vectors G at a time: loads them, adds the noise and
-// stores them.
-template <class Io, bool kTwo, bool kSame, bool kUniformHi, int G>
-__device__ __forceinline__ void axpy_tile(const TileRef<Io>& r, PhiloxKey key, float scale,
-                                          PhiloxKey key2, float scale2) {
-  constexpr int V = Io::kVec;
-  // the two-seed pass is fastest fully packed, the one-seed pass scalar
-  constexpr NoiseForm kAxpyForm = kTwo ? NoiseForm::kPacked : NoiseForm::kScalar;
-  typename Io::Scalar* const base = r.base;
-  const uint64_t numel = r.numel, index_base = r.index_base, t0 = r.t0;
-  const uint32_t j_hi = static_cast<uint32_t>((index_base + t0) >> 34);
-  const auto gen = make_gen<kUniformHi>(key, j_hi);
-  const auto gen2 = make_gen<kUniformHi && kTwo && !kSame>(key2, j_hi);
-#pragma unroll 1
-  for (int u0 = 0; u0 < kVecsPerThread; u0 += G) {
-    uint4 v[G];
+// First element of the calling thread's vector u of a tile. Vector u of a
+// tile is 256 consecutive 16-byte vectors, one per thread: each load and
+// store instruction of a warp covers 512 contiguous bytes.
+template <class Io>
+__device__ __forceinline__ uint64_t vec_elem(const TileRef<Io>& r, int u) {
+  return r.t0 + static_cast<uint64_t>(u * kBlockThreads + threadIdx.x) * Io::kVec;
+}
+
+// Vectors u0 .. u0 + G - 1 of the calling thread: a 16-byte load each; the
+// ragged end of a segment element by element, zeros past it.
+template <class Io, int G>
+__device__ __forceinline__ void load_group(const TileRef<Io>& r, int u0, uint4 (&v)[G]) {
 #pragma unroll
-    for (int u = 0; u < G; ++u) {
-      const uint64_t e = t0 + static_cast<uint64_t>((u0 + u) * kBlockThreads + threadIdx.x) * V;
-      v[u] = make_uint4(0u, 0u, 0u, 0u);
-      if (e + V <= numel) v[u] = *reinterpret_cast<const uint4*>(base + e);
+  for (int q = 0; q < G; ++q) {
+    const uint64_t e = vec_elem(r, u0 + q);
+    v[q] = make_uint4(0u, 0u, 0u, 0u);
+    if (e + Io::kVec <= r.numel)
+      v[q] = *reinterpret_cast<const uint4*>(r.base + e);
+    else if (e < r.numel)
+      v[q] = Io::load_partial(r.base, e, static_cast<int>(r.numel - e));
+  }
+}
+
+template <class Io>
+__device__ __forceinline__ void store_vec(const TileRef<Io>& r, uint64_t e, const uint4& v) {
+  if (e + Io::kVec <= r.numel)
+    *reinterpret_cast<uint4*>(r.base + e) = v;
+  else if (e < r.numel)
+    Io::store_partial(r.base, e, static_cast<int>(r.numel - e), v);
+}
+
+// Arguments of a perturb/restore launch: the schedule and scale of each step
+// (step 2 only with kTwo). A __grid_constant__ parameter, so every round key
+// is read from the constant bank as an instruction operand.
+struct AxpyArgs {
+  PhiloxSched s1, s2;
+  float scale1, scale2;
+};
+
+// One tile of the perturb/restore pass (kTwo: fused restore + perturb; kSame:
+// both steps use one seed, whose noise is generated once), G vectors at a
+// time. The loads of the next group (at the last group: the first group of
+// the CTA's next tile, `next`) are issued before the current group is
+// computed, so the memory latency hides behind the generator's work.
+template <class Io, bool kTwo, bool kSame, bool kUniformHi, int G>
+__device__ __forceinline__ void axpy_tile(const TileRef<Io>& cur, uint4 (&v)[G],
+                                          const AxpyArgs& a, const SegDesc* __restrict__ segs,
+                                          const float* __restrict__ inv_scale, int& seg,
+                                          uint64_t next, bool has_next, TileRef<Io>& nxt) {
+  constexpr int V = Io::kVec;
+  constexpr NoiseForm kAxpyForm = kTwo ? kAxpy2Form : kAxpy1Form;
+  constexpr int kGroups = kVecsPerThread / G;
+  const uint32_t j_hi = static_cast<uint32_t>((cur.index_base + cur.t0) >> 34);
+  const auto gen = sched_gen<kUniformHi>(a.s1, j_hi);
+  const auto gen2 = sched_gen<kUniformHi && kTwo && !kSame>(a.s2, j_hi);
+  const float s1 = a.scale1 * cur.inv, s2 = a.scale2 * cur.inv;
+#pragma unroll
+  for (int grp = 0; grp < kGroups; ++grp) {
+    uint4 nv[G];
+    if (grp + 1 < kGroups) {
+      load_group<Io, G>(cur, (grp + 1) * G, nv);
+    } else if (has_next) {
+      nxt = tile_ref<Io>(segs, inv_scale, seg, next);
+      load_group<Io, G>(nxt, 0, nv);
     }
 #pragma unroll
-    for (int u = 0; u < G; ++u) {
-      const uint64_t e = t0 + static_cast<uint64_t>((u0 + u) * kBlockThreads + threadIdx.x) * V;
-      if (e >= numel) continue;
-      const bool full = e + V <= numel;
-      const int rem = full ? V : static_cast<int>(numel - e);
+    for (int q = 0; q < G; ++q) {
+      const uint64_t e = vec_elem(cur, grp * G + q);
+      if (e >= cur.numel) continue;
       float f[V];
-      if (full) {
-        Io::unpack(v[u], f);
-      } else {  // ragged end of a segment
-#pragma unroll
-        for (int k = 0; k < V; ++k) f[k] = k < rem ? Io::to_f32(base[e + k]) : 0.0f;
-      }
-      if (kSame) {
-        add_scaled_noise_twice<Io, V>(gen, index_base + e, scale, scale2, f);
+      Io::unpack(v[q], f);
+      if constexpr (kSame) {
+        add_scaled_noise_twice<Io, V>(gen, cur.index_base + e, s1, s2, f);
       } else {
-        add_scaled_noise<kAxpyForm, V>(gen, index_base + e, scale, f);
-        if (kTwo) {
+        add_scaled_noise<kAxpyForm, V>(gen, cur.index_base + e, s1, f);
+        if constexpr (kTwo) {
           Io::round_trip(f);
-          add_scaled_noise<kAxpyForm, V>(gen2, index_base + e, scale2, f);
+          add_scaled_noise<kAxpyForm, V>(gen2, cur.index_base + e, s2, f);
         }
       }
-      if (full) {
-        *reinterpret_cast<uint4*>(base + e) = Io::pack(f);
-      } else {
+      store_vec(cur, e, Io::pack(f));
+    }
+    if (grp + 1 < kGroups || has_next) {
 #pragma unroll
-        for (int k = 0; k < V; ++k)
-          if (k < rem) base[e + k] = Io::from_f32(f[k]);
-      }
+      for (int q = 0; q < G; ++q) v[q] = nv[q];
     }
   }
 }
@@ -367,221 +415,217 @@ __device__ __forceinline__ void axpy_tile(const TileRef<Io>& r, PhiloxKey key, f
 template <class Io, bool kTwo, bool kSame>
 __global__ void __launch_bounds__(kBlockThreads, axpy_min_blocks(kTwo))
 axpy_noise_kernel(const SegDesc* __restrict__ segs, const float* __restrict__ inv_scale,
-                  uint64_t total_tiles, PhiloxKey key, float scale, PhiloxKey key2,
-                  float scale2) {
-  constexpr uint64_t kTile = static_cast<uint64_t>(kBlockThreads) * kVecsPerThread * Io::kVec;
+                  uint64_t total_tiles, const __grid_constant__ AxpyArgs a) {
   constexpr int G = group_for<Io>(kTwo ? kAxpy2Group : kAxpy1Group);
+  uint64_t tile = blockIdx.x;
+  if (tile >= total_tiles) return;
   int seg = 0;
-  for (uint64_t tile = blockIdx.x; tile < total_tiles; tile += gridDim.x) {
-    const TileRef<Io> cur = tile_ref<Io>(segs, seg, tile, kTile);
-    float s1 = scale, s2 = scale2;
-    if constexpr (Io::kScaled) {
-      const float inv = inv_scale[seg];
-      s1 *= inv;
-      s2 *= inv;
-    }
-    if (uniform_hi(cur.index_base, cur.t0, kTile, cur.numel))
-      axpy_tile<Io, kTwo, kSame, true, G>(cur, key, s1, key2, s2);
+  TileRef<Io> cur = tile_ref<Io>(segs, inv_scale, seg, tile);
+  uint4 v[G];
+  load_group<Io, G>(cur, 0, v);
+  for (;;) {
+    const uint64_t next = tile + gridDim.x;
+    const bool has_next = next < total_tiles;
+    TileRef<Io> nxt = cur;
+    if (uniform_hi(cur.index_base, cur.t0, static_cast<uint64_t>(kBlockThreads) * kVecsPerThread * Io::kVec, cur.numel))
+      axpy_tile<Io, kTwo, kSame, true, G>(cur, v, a, segs, inv_scale, seg, next, has_next, nxt);
     else
-      axpy_tile<Io, kTwo, kSame, false, G>(cur, key, s1, key2, s2);
+      axpy_tile<Io, kTwo, kSame, false, G>(cur, v, a, segs, inv_scale, seg, next, has_next, nxt);
+    if (!has_next) break;
+    tile = next;
+    cur = nxt;
   }
 }
 
-// One tile of a single-generation update (es_update; with kPerturb also the
-// trailing perturb of es_update_perturb): acc = sum_i c_i eps_i (fp32,
-// ascending i), then theta + acc rounded once (then + pscale * eps_pseed,
-// rounded again); theta read and written once. Vectors G at a time.
-template <class Io, bool kUniformHi, bool kPerturb, int G>
-__device__ __forceinline__ void update_tile_single(typename Io::Scalar* base, uint64_t numel,
-                                                   uint64_t index_base, uint64_t t0,
-                                                   const UpdateArgs& args, const PhiloxKey* s_key,
-                                                   const float* s_coeff, float inv) {
+// Seeds of an update launch are staged in shared memory kSchedRows at a time,
+// one row of kRowVecs 16-byte words per seed, filled by the CTA for the
+// high counter word j_hi of the tile at hand:
+//   row[0] = (k0, k1, round 1's k0, tile constant x2)
+//   row[1] = (tile constant lo2, coefficient bits, 0, 0)
+//   row[2 .. 5] = round keys of rounds 2..9
+// so a seed costs its thread six shared-memory loads instead of deriving its
+// key schedule and tile constants. Row kSchedRows is the trailing perturb's.
+constexpr int kSchedRows = 128;
+constexpr int kRowVecs = 6;
+using SchedRow = uint4[kRowVecs];
+
+__device__ __forceinline__ void fill_row(SchedRow& row, uint32_t k0, uint32_t k1, float coeff,
+                                         uint32_t j_hi) {
+  const PhiloxSched s = philox_sched(static_cast<uint64_t>(k1) << 32 | k0);
+  const TileConst t = tile_const(j_hi, s.rk[0], s.rk[3]);
+  row[0] = make_uint4(s.rk[0], s.rk[1], s.rk[2], t.x2);
+  row[1] = make_uint4(t.lo2, __float_as_uint(coeff), 0u, 0u);
+#pragma unroll
+  for (int k = 0; k < 4; ++k)
+    row[2 + k] = make_uint4(s.rk[4 + 4 * k], s.rk[5 + 4 * k], s.rk[6 + 4 * k], s.rk[7 + 4 * k]);
+}
+
+// Round keys of rounds 2..9 held in registers.
+struct KeyRegs {
+  uint32_t k[16];
+  __device__ uint32_t operator[](int i) const { return k[i]; }
+};
+
+// Generator and coefficient of one staged row.
+template <bool kUniformHi>
+__device__ __forceinline__ auto row_gen(const SchedRow& row) {
+  const uint4 r0 = row[0], r1 = row[1];
+  if constexpr (kUniformHi) {
+    KeyRegs kr;
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+      const uint4 w = row[2 + k];
+      kr.k[4 * k] = w.x;
+      kr.k[4 * k + 1] = w.y;
+      kr.k[4 * k + 2] = w.z;
+      kr.k[4 * k + 3] = w.w;
+    }
+    return SchedGen<KeyRegs>{TileConst{r0.w, r1.x}, r0.y, r0.z, kr};
+  } else {
+    return AnyGen{PhiloxKey{r0.x, r0.y}};
+  }
+}
+
+__device__ __forceinline__ float row_coeff(const SchedRow& row) { return __uint_as_float(row[1].y); }
+
+// Which seeds the CTA's rows hold, and for which j_hi.
+struct RowState {
+  int first;
+  uint32_t j_hi;
+};
+
+// Makes the rows hold seeds [c0, c0 + kSchedRows) (and the perturb row) for
+// j_hi. Called by every thread of the CTA with the same arguments.
+template <bool kPerturb>
+__device__ __forceinline__ void ensure_rows(SchedRow* s_rows, RowState& rs, const UpdateArgs& args,
+                                            int c0, uint32_t j_hi) {
+  if (rs.first == c0 && rs.j_hi == j_hi) return;
+  __syncthreads();  // every thread is done with the rows held so far
+  const int m = args.n - c0 < kSchedRows ? args.n - c0 : kSchedRows;
+  for (int k = threadIdx.x; k < m; k += kBlockThreads)
+    fill_row(s_rows[k], args.key[c0 + k][0], args.key[c0 + k][1], args.coeff[c0 + k], j_hi);
+  if (kPerturb && threadIdx.x == kBlockThreads - 1)
+    fill_row(s_rows[kSchedRows], args.pkey[0], args.pkey[1], args.pscale, j_hi);
+  __syncthreads();
+  rs.first = c0;
+  rs.j_hi = j_hi;
+}
+
+// acc[q] += c_i eps_i over the seeds i of [c0, c1) held in the rows from c0,
+// for the thread's vectors u0 .. u0 + G - 1 (ascending i).
+template <class Io, bool kUniformHi, int G>
+__device__ __forceinline__ void accumulate_seeds(const TileRef<Io>& r, int u0, const SchedRow* rows,
+                                                 int count, float (&acc)[G][Io::kVec]) {
   constexpr int V = Io::kVec;
   constexpr int kUnroll = ES_SEED_UNROLL;
-  const uint32_t j_hi = static_cast<uint32_t>((index_base + t0) >> 34);
+#pragma unroll kUnroll
+  for (int i = 0; i < count; ++i) {
+    const auto gen = row_gen<kUniformHi>(rows[i]);
+    const float c = row_coeff(rows[i]);
+#pragma unroll
+    for (int q = 0; q < G; ++q) {
+      const uint64_t e = vec_elem(r, u0 + q);
+      if (e >= r.numel) continue;
+      add_scaled_noise<kUpdateForm, V>(gen, r.index_base + e, c, acc[q]);
+    }
+  }
+}
+
+// v[q] <- round(v[q] + acc[q]) in storage form; acc <- 0.
+template <class Io, int G>
+__device__ __forceinline__ void apply_acc(uint4 (&v)[G], float (&acc)[G][Io::kVec], float inv) {
+#pragma unroll
+  for (int q = 0; q < G; ++q) {
+    float f[Io::kVec];
+    Io::unpack(v[q], f);
+#pragma unroll
+    for (int k = 0; k < Io::kVec; ++k) {
+      f[k] = add_acc<Io>(f[k], acc[q][k], inv);
+      acc[q][k] = 0.0f;
+    }
+    v[q] = Io::pack(f);
+  }
+}
+
+// One tile of a fused update launch, G vectors at a time. Theta stays in
+// registers in storage form; generation g adds acc_g = sum_{i in g} c_i eps_i
+// (fp32, ascending i) and rounds once, exactly as a separate launch per
+// generation would store it (kSingle: one generation, and with kPerturb the
+// next generation's first perturb follows, rounded again). Theta is read and
+// written once.
+template <class Io, bool kUniformHi, bool kSingle, bool kPerturb, int G>
+__device__ __forceinline__ void update_tile(const TileRef<Io>& r, const UpdateArgs& args,
+                                            SchedRow* s_rows, RowState& rs) {
+  constexpr int V = Io::kVec;
+  const uint32_t j_hi = static_cast<uint32_t>((r.index_base + r.t0) >> 34);
   const int n = args.n;
-  const float pscale = Io::kScaled ? args.pscale * inv : args.pscale;
-  const auto pgen = make_gen<kUniformHi && kPerturb>(PhiloxKey{args.pkey[0], args.pkey[1]}, j_hi);
 #pragma unroll 1
   for (int u0 = 0; u0 < kVecsPerThread; u0 += G) {
     uint4 v[G];
-#pragma unroll
-    for (int q = 0; q < G; ++q) {
-      const uint64_t e = t0 + static_cast<uint64_t>((u0 + q) * kBlockThreads + threadIdx.x) * V;
-      v[q] = make_uint4(0u, 0u, 0u, 0u);
-      if (e + V <= numel) v[q] = *reinterpret_cast<const uint4*>(base + e);
-    }
+    load_group<Io, G>(r, u0, v);
     float acc[G][V];
 #pragma unroll
     for (int q = 0; q < G; ++q)
 #pragma unroll
       for (int k = 0; k < V; ++k) acc[q][k] = 0.0f;
-#pragma unroll kUnroll
-    for (int i = 0; i < n; ++i) {
-      const auto gen = make_gen<kUniformHi>(s_key[i], j_hi);
-      const float c = s_coeff[i];
-#pragma unroll
-      for (int q = 0; q < G; ++q) {
-        const uint64_t e = t0 + static_cast<uint64_t>((u0 + q) * kBlockThreads + threadIdx.x) * V;
-        if (e >= numel) continue;
-        add_scaled_noise<NoiseForm::kPackedFma, V>(gen, index_base + e, c, acc[q]);
-      }
-    }
-#pragma unroll
-    for (int q = 0; q < G; ++q) {
-      const uint64_t e = t0 + static_cast<uint64_t>((u0 + q) * kBlockThreads + threadIdx.x) * V;
-      if (e >= numel) continue;
-      const bool full = e + V <= numel;
-      const int rem = full ? V : static_cast<int>(numel - e);
-      float f[V];
-      if (full) {
-        Io::unpack(v[q], f);
+    int g = 0;
+#pragma unroll 1
+    for (int c0 = 0; c0 < n; c0 += kSchedRows) {
+      ensure_rows<kPerturb>(s_rows, rs, args, c0, j_hi);
+      const int c1 = n - c0 < kSchedRows ? n : c0 + kSchedRows;
+      if constexpr (kSingle) {
+        accumulate_seeds<Io, kUniformHi, G>(r, u0, s_rows, c1 - c0, acc);
       } else {
-#pragma unroll
-        for (int k = 0; k < V; ++k) f[k] = k < rem ? Io::to_f32(base[e + k]) : 0.0f;
-      }
-#pragma unroll
-      for (int k = 0; k < V; ++k) f[k] = add_acc<Io>(f[k], acc[q][k], inv);
-      if (kPerturb) {
-        Io::round_trip(f);
-        add_scaled_noise<NoiseForm::kPackedFma, V>(pgen, index_base + e, pscale, f);
-      }
-      if (full) {
-        *reinterpret_cast<uint4*>(base + e) = Io::pack(f);
-      } else {
-#pragma unroll
-        for (int k = 0; k < V; ++k)
-          if (k < rem) base[e + k] = Io::from_f32(f[k]);
-      }
-    }
-  }
-}
-
-// One tile of a fused update launch. Theta stays in registers in storage
-// form; generation g adds acc_g = sum_{i in g} c_i eps_i (fp32, ascending i)
-// and rounds once, exactly as a separate launch per generation would store it;
-// an optional trailing perturb step follows. Theta is read and written once.
-// Vectors G at a time; lanes past the segment's end hold zeros and are never
-// stored.
-template <class Io, bool kUniformHi, int G>
-__device__ __forceinline__ void update_tile(typename Io::Scalar* base, uint64_t numel,
-                                            uint64_t index_base, uint64_t t0,
-                                            const UpdateArgs& args, const PhiloxKey* s_key,
-                                            const float* s_coeff, const uint16_t* s_gen_end,
-                                            float inv) {
-  constexpr int V = Io::kVec;
-  const uint32_t j_hi = static_cast<uint32_t>((index_base + t0) >> 34);
-#pragma unroll 1
-  for (int u0 = 0; u0 < kVecsPerThread; u0 += G) {
-    uint4 v[G];
-#pragma unroll
-    for (int q = 0; q < G; ++q) {
-      const uint64_t e = t0 + static_cast<uint64_t>((u0 + q) * kBlockThreads + threadIdx.x) * V;
-      v[q] = make_uint4(0u, 0u, 0u, 0u);
-      if (e + V <= numel)
-        v[q] = *reinterpret_cast<const uint4*>(base + e);
-      else if (e < numel)
-        v[q] = Io::load_partial(base, e, static_cast<int>(numel - e));
-    }
-    int i = 0;
-#pragma unroll 1
-    for (int g = 0; g < args.n_gen; ++g) {
-      float acc[G][V];
-#pragma unroll
-      for (int q = 0; q < G; ++q)
-#pragma unroll
-        for (int k = 0; k < V; ++k) acc[q][k] = 0.0f;
-      const int end = s_gen_end[g];
-#pragma unroll 1
-      for (; i < end; ++i) {
-        const auto gen = make_gen<kUniformHi>(s_key[i], j_hi);
-        const float c = s_coeff[i];
-#pragma unroll
-        for (int q = 0; q < G; ++q) {
-          const uint64_t e = t0 + static_cast<uint64_t>((u0 + q) * kBlockThreads + threadIdx.x) * V;
-          if (e >= numel) continue;
-          add_scaled_noise<NoiseForm::kPackedFma, V>(gen, index_base + e, c, acc[q]);
+        // generation by generation within the chunk (generations are never empty)
+        int i = c0;
+        while (i < c1) {
+          const int end = args.gen_end[g] < c1 ? args.gen_end[g] : c1;
+          accumulate_seeds<Io, kUniformHi, G>(r, u0, s_rows + (i - c0), end - i, acc);
+          i = end;
+          if (i == args.gen_end[g]) {
+            apply_acc<Io, G>(v, acc, r.inv);
+            ++g;
+          }
         }
       }
-#pragma unroll
-      for (int q = 0; q < G; ++q) {
-        float f[V];
-        Io::unpack(v[q], f);
-#pragma unroll
-        for (int k = 0; k < V; ++k) f[k] = add_acc<Io>(f[k], acc[q][k], inv);
-        v[q] = Io::pack(f);
-      }
     }
-    if (args.perturb) {
-      const auto gen = make_gen<kUniformHi>(PhiloxKey{args.pkey[0], args.pkey[1]}, j_hi);
+    if constexpr (kSingle) apply_acc<Io, G>(v, acc, r.inv);
+    if constexpr (kPerturb) {
+      const auto pgen = row_gen<kUniformHi>(s_rows[kSchedRows]);
+      const float ps = row_coeff(s_rows[kSchedRows]) * r.inv;
 #pragma unroll
       for (int q = 0; q < G; ++q) {
-        const uint64_t e = t0 + static_cast<uint64_t>((u0 + q) * kBlockThreads + threadIdx.x) * V;
-        if (e >= numel) continue;
+        const uint64_t e = vec_elem(r, u0 + q);
+        if (e >= r.numel) continue;
         float f[V];
         Io::unpack(v[q], f);
-        add_scaled_noise<NoiseForm::kPackedFma, V>(gen, index_base + e,
-                                                   Io::kScaled ? args.pscale * inv : args.pscale, f);
+        add_scaled_noise<kUpdateForm, V>(pgen, r.index_base + e, ps, f);
         v[q] = Io::pack(f);
       }
     }
 #pragma unroll
-    for (int q = 0; q < G; ++q) {
-      const uint64_t e = t0 + static_cast<uint64_t>((u0 + q) * kBlockThreads + threadIdx.x) * V;
-      if (e + V <= numel)
-        *reinterpret_cast<uint4*>(base + e) = v[q];
-      else if (e < numel)
-        Io::store_partial(base, e, static_cast<int>(numel - e), v[q]);
-    }
+    for (int q = 0; q < G; ++q) store_vec(r, vec_elem(r, u0 + q), v[q]);
   }
 }
 
 // Fused update launch (es_update, es_replay, es_update_perturb): for each
 // generation g, theta[g] <- round(theta[g] + sum_{i in g} c_i eps_{s_i}[g]),
-// then optionally theta <- round(theta + pscale * eps_pseed).
-// kSingle: one generation (update_tile_single, with a trailing perturb when
-// kPerturb); otherwise the general form (update_tile).
+// then with kPerturb theta <- round(theta + pscale * eps_pseed).
+// kSingle: one generation; otherwise args.n_gen generations, never empty.
 template <class Io, bool kSingle, bool kPerturb>
 __global__ void __launch_bounds__(kBlockThreads, update_min_blocks())
 update_kernel(const SegDesc* __restrict__ segs, const float* __restrict__ inv_scale,
               uint64_t total_tiles, const __grid_constant__ UpdateArgs args) {
-  constexpr uint64_t kTile = static_cast<uint64_t>(kBlockThreads) * kVecsPerThread * Io::kVec;
   constexpr int G = group_for<Io>(kUpdateGroup);
-  using S = typename Io::Scalar;
-  __shared__ PhiloxKey s_key[ES_MAX_SEEDS];
-  __shared__ float s_coeff[ES_MAX_SEEDS];
-  __shared__ uint16_t s_gen_end[kMaxGenerations];
-  for (int i = threadIdx.x; i < args.n; i += blockDim.x) {
-    s_key[i] = PhiloxKey{args.key[i][0], args.key[i][1]};
-    s_coeff[i] = args.coeff[i];
-  }
-  for (int g = threadIdx.x; g < args.n_gen; g += blockDim.x) s_gen_end[g] = args.gen_end[g];
-  __syncthreads();
-
+  __shared__ SchedRow s_rows[kSchedRows + 1];
+  RowState rs{-1, 0u};
   int seg = 0;
   for (uint64_t tile = blockIdx.x; tile < total_tiles; tile += gridDim.x) {
-    const SegDesc* d = find_segment(segs, seg, tile);
-    S* const base = static_cast<S*>(d->data);
-    const uint64_t numel = d->numel;
-    const uint64_t index_base = d->index_base;
-    const uint64_t t0 = (tile - d->tile_begin) * kTile;
-    const bool uhi = uniform_hi(index_base, t0, kTile, numel);
-    const float inv = Io::kScaled ? inv_scale[seg] : 1.0f;
-    if constexpr (kSingle) {
-      if (uhi)
-        update_tile_single<Io, true, kPerturb, G>(base, numel, index_base, t0, args, s_key,
-                                                  s_coeff, inv);
-      else
-        update_tile_single<Io, false, kPerturb, G>(base, numel, index_base, t0, args, s_key,
-                                                   s_coeff, inv);
-    } else {
-      if (uhi)
-        update_tile<Io, true, G>(base, numel, index_base, t0, args, s_key, s_coeff, s_gen_end,
-                                 inv);
-      else
-        update_tile<Io, false, G>(base, numel, index_base, t0, args, s_key, s_coeff, s_gen_end,
-                                  inv);
-    }
+    const TileRef<Io> r = tile_ref<Io>(segs, inv_scale, seg, tile);
+    if (uniform_hi(r.index_base, r.t0, static_cast<uint64_t>(kBlockThreads) * kVecsPerThread * Io::kVec, r.numel))
+      update_tile<Io, true, kSingle, kPerturb, G>(r, args, s_rows, rs);
+    else
+      update_tile<Io, false, kSingle, kPerturb, G>(r, args, s_rows, rs);
   }
 }
 
@@ -711,39 +755,37 @@ int persistent_grid(K kernel, uint64_t work_items) {
 }
 
 template <class Io, bool kTwo, bool kSame>
-cudaError_t launch_axpy_io(const PlanView& plan, PhiloxKey key, float scale, PhiloxKey key2,
-                           float scale2, cudaStream_t stream) {
+cudaError_t launch_axpy_io(const PlanView& plan, const AxpyArgs& a, cudaStream_t stream) {
   auto k = axpy_noise_kernel<Io, kTwo, kSame>;
   k<<<persistent_grid(k, plan.total_tiles), kBlockThreads, 0, stream>>>(
-      plan.segs, plan.inv_scale, plan.total_tiles, key, scale, key2, scale2);
+      plan.segs, plan.inv_scale, plan.total_tiles, a);
   return cudaGetLastError();
 }
 
 template <bool kTwo, bool kSame>
-cudaError_t launch_axpy(const PlanView& plan, PhiloxKey key, float scale, PhiloxKey key2,
+cudaError_t launch_axpy(const PlanView& plan, uint64_t seed, float scale, uint64_t seed2,
                         float scale2, cudaStream_t stream) {
-  if (plan.dtype == ES_BF16)
-    return launch_axpy_io<Bf16Io, kTwo, kSame>(plan, key, scale, key2, scale2, stream);
-  if (plan.dtype == ES_FP8_E4M3)
-    return launch_axpy_io<Fp8Io, kTwo, kSame>(plan, key, scale, key2, scale2, stream);
-  return launch_axpy_io<F32Io, kTwo, kSame>(plan, key, scale, key2, scale2, stream);
+  AxpyArgs a;
+  a.s1 = philox_sched(seed);
+  a.s2 = philox_sched(seed2);
+  a.scale1 = scale;
+  a.scale2 = scale2;
+  if (plan.dtype == ES_BF16) return launch_axpy_io<Bf16Io, kTwo, kSame>(plan, a, stream);
+  if (plan.dtype == ES_FP8_E4M3) return launch_axpy_io<Fp8Io, kTwo, kSame>(plan, a, stream);
+  return launch_axpy_io<F32Io, kTwo, kSame>(plan, a, stream);
 }
 
 }  // namespace
 
 cudaError_t launch_axpy_noise(const PlanView& plan, uint64_t seed, float scale,
                               cudaStream_t stream) {
-  return launch_axpy<false, false>(plan, philox_key(seed), scale, PhiloxKey{0u, 0u}, 0.0f,
-                                   stream);
+  return launch_axpy<false, false>(plan, seed, scale, 0u, 0.0f, stream);
 }
 
 cudaError_t launch_axpy_noise2(const PlanView& plan, uint64_t seed, float scale, uint64_t seed2,
                                float scale2, cudaStream_t stream) {
-  if (seed == seed2)
-    return launch_axpy<true, true>(plan, philox_key(seed), scale, philox_key(seed2), scale2,
-                                   stream);
-  return launch_axpy<true, false>(plan, philox_key(seed), scale, philox_key(seed2), scale2,
-                                  stream);
+  if (seed == seed2) return launch_axpy<true, true>(plan, seed, scale, seed2, scale2, stream);
+  return launch_axpy<true, false>(plan, seed, scale, seed2, scale2, stream);
 }
 
 template <class Io>

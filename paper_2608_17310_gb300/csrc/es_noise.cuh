@@ -115,6 +115,66 @@ __device__ __forceinline__ uint4 philox_block_tile(uint32_t j_lo, const PhiloxTi
   return make_uint4(c0, c1, c2, c3);
 }
 
+// The key schedule of one seed, computed once on the host or per CTA:
+// rk[2r] = k0 + r W_A and rk[2r + 1] = k1 + r W_B are the keys of round r
+// (r = 0..9). A kernel that takes it reads every round key as an operand
+// instead of deriving it, so the schedule costs no instruction per block.
+struct PhiloxSched {
+  uint32_t rk[20];
+};
+
+__host__ __device__ inline PhiloxSched philox_sched(uint64_t seed) {
+  PhiloxSched s;
+  uint32_t k0 = static_cast<uint32_t>(seed), k1 = static_cast<uint32_t>(seed >> 32);
+  for (int r = 0; r < 10; ++r) {
+    s.rk[2 * r] = k0;
+    s.rk[2 * r + 1] = k1;
+    k0 += kPhiloxWeylA;
+    k1 += kPhiloxWeylB;
+  }
+  return s;
+}
+
+// Per-tile constants of philox_tile, from a schedule: word 0 after round 0
+// is j_hi ^ k0, and round 1's product of it is shared by every block whose
+// counter has high word j_hi.
+struct TileConst {
+  uint32_t x2;   // high word of kPhiloxMulA * (j_hi ^ k0), xored with round 1's k1
+  uint32_t lo2;  // low word of kPhiloxMulA * (j_hi ^ k0)
+};
+
+__device__ __forceinline__ TileConst tile_const(uint32_t j_hi, uint32_t k0, uint32_t k1_round1) {
+  const uint32_t w0 = j_hi ^ k0;
+  return TileConst{mul_hi(kPhiloxMulA, w0) ^ k1_round1, mul_lo(kPhiloxMulA, w0)};
+}
+
+// philox_block_tile with the round keys taken from a schedule: `rk1` is round
+// 0's k1, `rk2` round 1's k0, `rk` points at the keys of rounds 2..9 (rk[2r - 4],
+// rk[2r - 3] for round r). Bit-identical to philox_block.
+template <class Keys>
+__device__ __forceinline__ uint4 philox_block_rk(uint32_t j_lo, TileConst t, uint32_t rk1,
+                                                 uint32_t rk2, const Keys& rk) {
+  const uint32_t a2 = mul_hi(kPhiloxMulA, j_lo) ^ rk1;  // round 0, word 2
+  const uint32_t a3 = mul_lo(kPhiloxMulA, j_lo);        // round 0, word 3
+  uint32_t c0 = mul_hi(kPhiloxMulB, a2) ^ rk2;          // round 1 (its word 1 was 0)
+  uint32_t c1 = mul_lo(kPhiloxMulB, a2);
+  uint32_t c2 = t.x2 ^ a3;
+  uint32_t c3 = t.lo2;
+#pragma unroll
+  for (int round = 2; round < 10; ++round) {
+    uint32_t ha, la, hb, lb;
+    mul_wide(kPhiloxMulA, c0, ha, la);
+    mul_wide(kPhiloxMulB, c2, hb, lb);
+    const uint32_t n0 = hb ^ c1 ^ rk[2 * round - 4];
+    const uint32_t n2 = ha ^ c3 ^ rk[2 * round - 3];
+    c1 = lb;
+    c3 = la;
+    c0 = n0;
+    c2 = n2;
+  }
+  return make_uint4(c0, c1, c2, c3);
+}
+
 // The float 1 + m 2^-23 for m = x >> 9 (the top 23 bits of x).
 __device__ __forceinline__ float one_plus_top23(uint32_t x) {
   return __uint_as_float(0x3F800000u | (x >> 9));

@@ -298,8 +298,12 @@ probe_kernel(int iters, uint32_t seed, unsigned long long* __restrict__ rec,
     unsigned long long n1;
     const unsigned long long c1 = clock64();
     asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(n1));
-    rec[2 * blockIdx.x] = c1 - c0;
-    rec[2 * blockIdx.x + 1] = n1 - n0;
+    unsigned int smid;
+    asm volatile("mov.u32 %0, %%smid;" : "=r"(smid));
+    rec[4 * blockIdx.x] = c0;
+    rec[4 * blockIdx.x + 1] = c1;
+    rec[4 * blockIdx.x + 2] = n1 - n0;
+    rec[4 * blockIdx.x + 3] = smid;
   }
   // Fold every chain into one word so that no chain is dead code; the store
   // happens only for a value that depends on all of them and the seed.
@@ -344,10 +348,13 @@ const char* esprobe_unit(int probe) {
 // Runs probe `probe` on the current device with ctas_per_sm CTAs of 256
 // threads on every SM (all resident at once; fewer if the probe's registers
 // allow fewer) for `iters` iterations, after one untimed launch.
-// out[0..6] = milliseconds (CUDA events), mean SM cycles per CTA, SM clock in
-// MHz (cycles / globaltimer ns), ops per clock per SM, ops in total, active
-// threads per SM, CTAs per SM used. Returns 0, -1 for a bad argument, else the
-// cudaError_t.
+// An SM's time is the span of its own SM clock (clock64) from the first of its
+// CTAs to start to the last to finish: the CTAs of one SM neither start nor end
+// together, so a CTA's own duration would overstate the SM's rate.
+// out[0..6] = milliseconds (CUDA events), mean SM cycles per SM (that span),
+// SM clock in MHz (CTA cycles / globaltimer ns), ops per clock per SM, ops in
+// total, active threads per SM, CTAs per SM used. Returns 0, -1 for a bad
+// argument, else the cudaError_t.
 int esprobe_run(int probe, int ctas_per_sm, int iters, double* out) {
   if (probe < 0 || probe >= kProbeCount || ctas_per_sm < 1 || iters < 1 || out == nullptr)
     return -1;
@@ -363,11 +370,11 @@ int esprobe_run(int probe, int ctas_per_sm, int iters, double* out) {
   unsigned long long* rec = nullptr;
   uint32_t* sink = nullptr;
   cudaEvent_t e0 = nullptr, e1 = nullptr;
-  err = cudaMalloc(&rec, sizeof(unsigned long long) * 2 * grid);
+  err = cudaMalloc(&rec, sizeof(unsigned long long) * 4 * grid);
   if (err == cudaSuccess) err = cudaMalloc(&sink, sizeof(uint32_t));
   if (err == cudaSuccess) err = cudaEventCreate(&e0);
   if (err == cudaSuccess) err = cudaEventCreate(&e1);
-  unsigned long long* host = new unsigned long long[2 * grid];
+  unsigned long long* host = new unsigned long long[4 * grid];
   float ms = 0.0f;
   if (err == cudaSuccess) {
     uint32_t seed = 0x51ED270Bu;
@@ -382,22 +389,46 @@ int esprobe_run(int probe, int ctas_per_sm, int iters, double* out) {
     if (err == cudaSuccess) err = cudaEventSynchronize(e1);
     if (err == cudaSuccess) err = cudaEventElapsedTime(&ms, e0, e1);
     if (err == cudaSuccess)
-      err = cudaMemcpy(host, rec, sizeof(unsigned long long) * 2 * grid, cudaMemcpyDeviceToHost);
+      err = cudaMemcpy(host, rec, sizeof(unsigned long long) * 4 * grid, cudaMemcpyDeviceToHost);
   }
   if (err == cudaSuccess) {
-    double cyc = 0.0, ns = 0.0;
-    for (int b = 0; b < grid; ++b) {
-      cyc += static_cast<double>(host[2 * b]);
-      ns += static_cast<double>(host[2 * b + 1]);
+    // per SM: [first start, last end] on its own clock (%smid may exceed the
+    // SM count: ids need not be contiguous)
+    constexpr int kMaxSmId = 4096;
+    unsigned long long* first = new unsigned long long[kMaxSmId];
+    unsigned long long* last = new unsigned long long[kMaxSmId];
+    for (int k = 0; k < kMaxSmId; ++k) {
+      first[k] = ~0ull;
+      last[k] = 0ull;
     }
-    cyc /= grid;
-    ns /= grid;
+    double cta_cyc = 0.0, ns = 0.0;
+    for (int b = 0; b < grid; ++b) {
+      const unsigned long long c0 = host[4 * b], c1 = host[4 * b + 1];
+      const int sm = static_cast<int>(host[4 * b + 3]);
+      cta_cyc += static_cast<double>(c1 - c0);
+      ns += static_cast<double>(host[4 * b + 2]);
+      if (sm >= 0 && sm < kMaxSmId) {
+        if (c0 < first[sm]) first[sm] = c0;
+        if (c1 > last[sm]) last[sm] = c1;
+      }
+    }
+    double cyc = 0.0;
+    int used = 0;
+    for (int k = 0; k < kMaxSmId; ++k)
+      if (last[k] > first[k]) {
+        cyc += static_cast<double>(last[k] - first[k]);
+        ++used;
+      }
+    const double sum_spans = cyc > 0.0 ? cyc : 1.0;
+    cyc = used > 0 ? cyc / used : 1.0;
+    delete[] first;
+    delete[] last;
     const double threads_per_sm = static_cast<double>(ctas_per_sm) * kThreads;
     const double ops = kInfo[probe].ops_per_iter * iters * threads_per_sm * kInfo[probe].active;
     out[0] = ms;
     out[1] = cyc;
-    out[2] = ns > 0.0 ? cyc / ns * 1e3 : 0.0;
-    out[3] = ops / cyc;
+    out[2] = ns > 0.0 ? cta_cyc / ns * 1e3 : 0.0;
+    out[3] = ops * sms / sum_spans;  // every CTA's ops over every SM's span
     out[4] = ops * sms;
     out[5] = threads_per_sm * kInfo[probe].active;
     out[6] = ctas_per_sm;
