@@ -23,10 +23,10 @@ constexpr int kVecsPerThread = 4;
 // of the compiler (a register cap), and the instruction form of the noise step
 // (0 scalar FP32, 1 scalar transform with packed FMAs, 2 packed; the values
 // are bit-identical). Measured on sm_103a over the 4B-shaped set: one vector
-// at a time at 3 CTAs per SM is fastest for every kernel; more CTAs per SM,
-// larger groups or a second seed in flight gain nothing, since the generator
-// is bound by the FMA-heavy pipe (its integer products and packed FP32), not
-// by latency.
+// at a time is fastest for every kernel, at 2 CTAs per SM (128 registers) for
+// the two-seed pass and 3 for the others; more CTAs per SM, larger groups or a
+// second seed in flight gain nothing, since the generator is bound by the
+// FMA-heavy pipe (its integer products and packed FP32), not by latency.
 #ifndef ES_AXPY1_GROUP
 #define ES_AXPY1_GROUP 1
 #endif
@@ -40,7 +40,7 @@ constexpr int kVecsPerThread = 4;
 #define ES_AXPY2_GROUP 1
 #endif
 #ifndef ES_AXPY2_MIN_BLOCKS
-#define ES_AXPY2_MIN_BLOCKS 3
+#define ES_AXPY2_MIN_BLOCKS 2
 #endif
 #ifndef ES_AXPY2_FORM
 #define ES_AXPY2_FORM 2

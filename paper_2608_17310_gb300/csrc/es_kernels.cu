@@ -219,14 +219,14 @@ constexpr NoiseForm kAxpy1Form = static_cast<NoiseForm>(ES_AXPY1_FORM);
 constexpr NoiseForm kAxpy2Form = static_cast<NoiseForm>(ES_AXPY2_FORM);
 constexpr NoiseForm kUpdateForm = static_cast<NoiseForm>(ES_UPDATE_FORM);
 
-// f[k] += scale * eps[g0 + k] for the V elements from global index g0
-// (g0 % 4 == 0), with scale folded into each pair's radius.
+// f[k] += scale * eps[4 j0 + k] for the V elements of Philox blocks j0,
+// j0 + 1, ..., with scale folded into each pair's radius.
 template <NoiseForm kForm, int V, class Gen>
-__device__ __forceinline__ void add_scaled_noise(const Gen& gen, uint64_t g0, float scale,
+__device__ __forceinline__ void add_scaled_noise(const Gen& gen, uint64_t j0, float scale,
                                                  float (&f)[V]) {
 #pragma unroll
   for (int b = 0; b < V / 4; ++b) {
-    const uint4 x = gen.block((g0 >> 2) + b);
+    const uint4 x = gen.block(j0 + b);
     if constexpr (kForm == NoiseForm::kScalar) {
       const Polar p = polar(x.x, x.y);
       const Polar q = polar(x.z, x.w);
@@ -259,11 +259,11 @@ __device__ __forceinline__ void add_scaled_noise(const Gen& gen, uint64_t g0, fl
 // f <- round(round(f + s1 * eps) + s2 * eps) for one seed's noise, computed
 // once: an antithetic restore (+eps out) followed by the perturb (-eps in).
 template <class Io, int V, class Gen>
-__device__ __forceinline__ void add_scaled_noise_twice(const Gen& gen, uint64_t g0, float s1,
+__device__ __forceinline__ void add_scaled_noise_twice(const Gen& gen, uint64_t j0, float s1,
                                                        float s2, float (&f)[V]) {
 #pragma unroll
   for (int b = 0; b < V / 4; ++b) {
-    const uint4 x = gen.block((g0 >> 2) + b);
+    const uint4 x = gen.block(j0 + b);
     const Polar p = polar(x.x, x.y);
     const Polar q = polar(x.z, x.w);
     float h[4];
@@ -359,8 +359,11 @@ struct AxpyArgs {
 // both steps use one seed, whose noise is generated once), G vectors at a
 // time. The loads of the next group (at the last group: the first group of
 // the CTA's next tile, `next`) are issued before the current group is
-// computed, so the memory latency hides behind the generator's work.
-template <class Io, bool kTwo, bool kSame, bool kUniformHi, int G>
+// computed, so the memory latency hides behind the generator's work. kFull:
+// the whole tile lies inside its segment (every tile but a segment's last),
+// so its vectors are addressed from one per-thread pointer and block index
+// without bounds checks.
+template <class Io, bool kTwo, bool kSame, bool kUniformHi, bool kFull, int G>
 __device__ __forceinline__ void axpy_tile(const TileRef<Io>& cur, uint4 (&v)[G],
                                           const AxpyArgs& a, const SegDesc* __restrict__ segs,
                                           const float* __restrict__ inv_scale, int& seg,
@@ -368,35 +371,52 @@ __device__ __forceinline__ void axpy_tile(const TileRef<Io>& cur, uint4 (&v)[G],
   constexpr int V = Io::kVec;
   constexpr NoiseForm kAxpyForm = kTwo ? kAxpy2Form : kAxpy1Form;
   constexpr int kGroups = kVecsPerThread / G;
+  constexpr int kStride = kBlockThreads * V;  // elements from one vector of a thread to the next
   const uint32_t j_hi = static_cast<uint32_t>((cur.index_base + cur.t0) >> 34);
   const auto gen = sched_gen<kUniformHi>(a.s1, j_hi);
   const auto gen2 = sched_gen<kUniformHi && kTwo && !kSame>(a.s2, j_hi);
   const float s1 = a.scale1 * cur.inv, s2 = a.scale2 * cur.inv;
+  // the thread's first element of the tile, and its Philox block (index_base
+  // is a multiple of 8 and t0 of the tile size, so the division is exact)
+  typename Io::Scalar* const p = cur.base + cur.t0 + threadIdx.x * V;
+  const uint64_t j_thread = ((cur.index_base + cur.t0) >> 2) + threadIdx.x * (V / 4);
 #pragma unroll
   for (int grp = 0; grp < kGroups; ++grp) {
     uint4 nv[G];
     if (grp + 1 < kGroups) {
-      load_group<Io, G>(cur, (grp + 1) * G, nv);
+      if constexpr (kFull) {
+#pragma unroll
+        for (int q = 0; q < G; ++q)
+          nv[q] = *reinterpret_cast<const uint4*>(p + ((grp + 1) * G + q) * kStride);
+      } else {
+        load_group<Io, G>(cur, (grp + 1) * G, nv);
+      }
     } else if (has_next) {
       nxt = tile_ref<Io>(segs, inv_scale, seg, next);
       load_group<Io, G>(nxt, 0, nv);
     }
 #pragma unroll
     for (int q = 0; q < G; ++q) {
-      const uint64_t e = vec_elem(cur, grp * G + q);
-      if (e >= cur.numel) continue;
+      const int u = grp * G + q;
+      if constexpr (!kFull) {
+        if (vec_elem(cur, u) >= cur.numel) continue;
+      }
+      const uint64_t j0 = j_thread + static_cast<uint64_t>(u) * (kStride / 4);
       float f[V];
       Io::unpack(v[q], f);
       if constexpr (kSame) {
-        add_scaled_noise_twice<Io, V>(gen, cur.index_base + e, s1, s2, f);
+        add_scaled_noise_twice<Io, V>(gen, j0, s1, s2, f);
       } else {
-        add_scaled_noise<kAxpyForm, V>(gen, cur.index_base + e, s1, f);
+        add_scaled_noise<kAxpyForm, V>(gen, j0, s1, f);
         if constexpr (kTwo) {
           Io::round_trip(f);
-          add_scaled_noise<kAxpyForm, V>(gen2, cur.index_base + e, s2, f);
+          add_scaled_noise<kAxpyForm, V>(gen2, j0, s2, f);
         }
       }
-      store_vec(cur, e, Io::pack(f));
+      if constexpr (kFull)
+        *reinterpret_cast<uint4*>(p + u * kStride) = Io::pack(f);
+      else
+        store_vec(cur, vec_elem(cur, u), Io::pack(f));
     }
     if (grp + 1 < kGroups || has_next) {
 #pragma unroll
@@ -427,10 +447,16 @@ axpy_noise_kernel(const SegDesc* __restrict__ segs, const float* __restrict__ in
     const uint64_t next = tile + gridDim.x;
     const bool has_next = next < total_tiles;
     TileRef<Io> nxt = cur;
-    if (uniform_hi(cur.index_base, cur.t0, static_cast<uint64_t>(kBlockThreads) * kVecsPerThread * Io::kVec, cur.numel))
-      axpy_tile<Io, kTwo, kSame, true, G>(cur, v, a, segs, inv_scale, seg, next, has_next, nxt);
+    constexpr uint64_t kTile = static_cast<uint64_t>(kBlockThreads) * kVecsPerThread * Io::kVec;
+    if (!uniform_hi(cur.index_base, cur.t0, kTile, cur.numel))
+      axpy_tile<Io, kTwo, kSame, false, false, G>(cur, v, a, segs, inv_scale, seg, next, has_next,
+                                                  nxt);
+    else if (cur.t0 + kTile <= cur.numel)
+      axpy_tile<Io, kTwo, kSame, true, true, G>(cur, v, a, segs, inv_scale, seg, next, has_next,
+                                                nxt);
     else
-      axpy_tile<Io, kTwo, kSame, false, G>(cur, v, a, segs, inv_scale, seg, next, has_next, nxt);
+      axpy_tile<Io, kTwo, kSame, true, false, G>(cur, v, a, segs, inv_scale, seg, next, has_next,
+                                                 nxt);
     if (!has_next) break;
     tile = next;
     cur = nxt;
@@ -526,7 +552,7 @@ __device__ __forceinline__ void accumulate_seeds(const TileRef<Io>& r, int u0, c
     for (int q = 0; q < G; ++q) {
       const uint64_t e = vec_elem(r, u0 + q);
       if (e >= r.numel) continue;
-      add_scaled_noise<kUpdateForm, V>(gen, r.index_base + e, c, acc[q]);
+      add_scaled_noise<kUpdateForm, V>(gen, (r.index_base + e) >> 2, c, acc[q]);
     }
   }
 }
@@ -599,7 +625,7 @@ __device__ __forceinline__ void update_tile(const TileRef<Io>& r, const UpdateAr
         if (e >= r.numel) continue;
         float f[V];
         Io::unpack(v[q], f);
-        add_scaled_noise<kUpdateForm, V>(pgen, r.index_base + e, ps, f);
+        add_scaled_noise<kUpdateForm, V>(pgen, (r.index_base + e) >> 2, ps, f);
         v[q] = Io::pack(f);
       }
     }
