@@ -99,6 +99,12 @@ void oracle_noise_block(uint64_t seed, uint64_t j, uint32_t out[4]) {
  * 32-bit output: u = (2 m + 1) / 2^24 with m = x >> 9. The set of values is
  * symmetric about 1/2 and excludes 0 and 1, so log(u) is always finite.
  */
+/* Words of blocks j0 .. j0 + n - 1, block after block (4 words each): the
+ * same definition as oracle_noise_block, over a range. */
+void oracle_noise_blocks(uint64_t seed, uint64_t j0, uint64_t n, uint32_t* out) {
+  for (uint64_t k = 0; k < n; ++k) oracle_noise_block(seed, j0 + k, out + 4 * k);
+}
+
 double oracle_uniform(uint32_t x) {
   double m = (double)(x >> 9);
   return (2.0 * m + 1.0) / 16777216.0;

@@ -52,6 +52,8 @@ def lib() -> ctypes.CDLL:
             L = ctypes.CDLL(build())
             L.oracle_philox4x32_10.argtypes = [_u32p, _u32p, _u32p]
             L.oracle_noise_block.argtypes = [ctypes.c_uint64, ctypes.c_uint64, _u32p]
+            L.oracle_noise_blocks.argtypes = [ctypes.c_uint64, ctypes.c_uint64, ctypes.c_uint64,
+                                              _u32p]
             L.oracle_uniform.argtypes = [ctypes.c_uint32]
             L.oracle_uniform.restype = ctypes.c_double
             L.oracle_box_muller_fill.argtypes = [_u32p, ctypes.c_uint64, _f64p]
@@ -119,6 +121,14 @@ def philox4x32_10(counter, key) -> np.ndarray:
 def noise_block(seed: int, j: int) -> np.ndarray:
     out = np.zeros(4, dtype=np.uint32)
     lib().oracle_noise_block(seed, j, _ptr(out, _u32p))
+    return out
+
+
+def noise_blocks(seed: int, j0: int, n: int) -> np.ndarray:
+    """Philox words of blocks j0 .. j0 + n - 1, shape (n, 4)."""
+    out = np.zeros((n, 4), dtype=np.uint32)
+    if n:
+        lib().oracle_noise_blocks(seed, j0, n, _ptr(out, _u32p))
     return out
 
 

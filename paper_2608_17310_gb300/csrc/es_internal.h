@@ -52,7 +52,14 @@ constexpr int kVecsPerThread = 4;
 #define ES_UPDATE_MIN_BLOCKS 3
 #endif
 #ifndef ES_UPDATE_FORM
-#define ES_UPDATE_FORM 1
+#define ES_UPDATE_FORM 2
+#endif
+// Radius inputs within 2^-10 of 1 (one in 1024), which take the series of
+// -2 ln u instead of the hardware log2: found by a compare on the raw Philox
+// word and fixed on a rarely taken branch (1), or by evaluating both forms
+// for every pair and selecting (0). The values are identical.
+#ifndef ES_NEAR_ONE_BRANCH
+#define ES_NEAR_ONE_BRANCH 1
 #endif
 // Seeds of the update's seed loop issued together (independent generator
 // work per element across seeds; the accumulation stays in ascending order).

@@ -218,31 +218,69 @@ enum class NoiseForm { kScalar, kPackedFma, kPacked };
 constexpr NoiseForm kAxpy1Form = static_cast<NoiseForm>(ES_AXPY1_FORM);
 constexpr NoiseForm kAxpy2Form = static_cast<NoiseForm>(ES_AXPY2_FORM);
 constexpr NoiseForm kUpdateForm = static_cast<NoiseForm>(ES_UPDATE_FORM);
+// Near-one radius inputs: a rare branch (true) or a select per pair (false).
+constexpr bool kNearOneBranch = ES_NEAR_ONE_BRANCH != 0;
+
+// Radius^2 of every pair of NB Philox blocks (p[b].r, from the hardware log2)
+// corrected where the radius input lies within 2^-10 of 1: such a pair takes
+// the series instead. The test is on the raw words (xa[b] = the blocks' words
+// x0 and x2), and the series is computed only when some pair needs it (one
+// radius input in 1024), so the common path costs one compare per pair. The
+// values equal radius_sq's.
+template <int NB>
+__device__ __forceinline__ void fix_near_one(const uint2 (&xa)[NB], Polar2 (&p)[NB]) {
+  bool near = false;
+#pragma unroll
+  for (int b = 0; b < NB; ++b) near |= (xa[b].x >= kNearOneWord) | (xa[b].y >= kNearOneWord);
+  if (__builtin_expect(near, 0)) {
+#pragma unroll
+    for (int b = 0; b < NB; ++b) {
+      if (xa[b].x >= kNearOneWord) p[b].r.x = radius_sq_series(uniform_open(xa[b].x));
+      if (xa[b].y >= kNearOneWord) p[b].r.y = radius_sq_series(uniform_open(xa[b].y));
+    }
+  }
+}
+
+// The pairs of Philox blocks j0 .. j0 + NB - 1 in polar form (r, cos, sin),
+// .x of each Polar2 the block's pair (x0, x1), .y its pair (x2, x3).
+template <NoiseForm kForm, int NB, class Gen>
+__device__ __forceinline__ void polar_blocks(const Gen& gen, uint64_t j0, Polar2 (&p)[NB]) {
+  constexpr bool kLogOnly = kNearOneBranch;
+  uint2 xa[NB];
+#pragma unroll
+  for (int b = 0; b < NB; ++b) {
+    const uint4 x = gen.block(j0 + b);
+    xa[b] = make_uint2(x.x, x.z);
+    if constexpr (kForm == NoiseForm::kPacked) {
+      p[b] = polar2_sq<kLogOnly>(x);
+    } else {
+      const Polar a = polar_sq<kLogOnly>(x.x, x.y), c = polar_sq<kLogOnly>(x.z, x.w);
+      p[b] = Polar2{make_float2(a.r, c.r), make_float2(a.c, c.c), make_float2(a.s, c.s)};
+    }
+  }
+  if constexpr (kLogOnly) fix_near_one<NB>(xa, p);
+#pragma unroll
+  for (int b = 0; b < NB; ++b) p[b].r = make_float2(sqrt_approx(p[b].r.x), sqrt_approx(p[b].r.y));
+}
 
 // f[k] += scale * eps[4 j0 + k] for the V elements of Philox blocks j0,
 // j0 + 1, ..., with scale folded into each pair's radius.
 template <NoiseForm kForm, int V, class Gen>
 __device__ __forceinline__ void add_scaled_noise(const Gen& gen, uint64_t j0, float scale,
                                                  float (&f)[V]) {
+  constexpr int NB = V / 4;
+  Polar2 pp[NB];
+  polar_blocks<kForm, NB>(gen, j0, pp);
 #pragma unroll
-  for (int b = 0; b < V / 4; ++b) {
-    const uint4 x = gen.block(j0 + b);
+  for (int b = 0; b < NB; ++b) {
+    const Polar2& p = pp[b];
     if constexpr (kForm == NoiseForm::kScalar) {
-      const Polar p = polar(x.x, x.y);
-      const Polar q = polar(x.z, x.w);
-      const float sp = -(scale * p.r), sq = -(scale * q.r);
-      f[4 * b + 0] = fmaf(sp, p.c, f[4 * b + 0]);
-      f[4 * b + 1] = fmaf(sp, p.s, f[4 * b + 1]);
-      f[4 * b + 2] = fmaf(sq, q.c, f[4 * b + 2]);
-      f[4 * b + 3] = fmaf(sq, q.s, f[4 * b + 3]);
+      const float sp = -(scale * p.r.x), sq = -(scale * p.r.y);
+      f[4 * b + 0] = fmaf(sp, p.c.x, f[4 * b + 0]);
+      f[4 * b + 1] = fmaf(sp, p.s.x, f[4 * b + 1]);
+      f[4 * b + 2] = fmaf(sq, p.c.y, f[4 * b + 2]);
+      f[4 * b + 3] = fmaf(sq, p.s.y, f[4 * b + 3]);
     } else {
-      Polar2 p;
-      if constexpr (kForm == NoiseForm::kPacked) {
-        p = polar2(x);
-      } else {
-        const Polar a = polar(x.x, x.y), c = polar(x.z, x.w);
-        p = Polar2{make_float2(a.r, c.r), make_float2(a.c, c.c), make_float2(a.s, c.s)};
-      }
       const float2 sr = __fmul2_rn(make_float2(-scale, -scale), p.r);   // -(scale * r)
       const float2 lo = __ffma2_rn(make_float2(sr.x, sr.x), make_float2(p.c.x, p.s.x),
                                    make_float2(f[4 * b + 0], f[4 * b + 1]));
@@ -261,21 +299,22 @@ __device__ __forceinline__ void add_scaled_noise(const Gen& gen, uint64_t j0, fl
 template <class Io, int V, class Gen>
 __device__ __forceinline__ void add_scaled_noise_twice(const Gen& gen, uint64_t j0, float s1,
                                                        float s2, float (&f)[V]) {
+  constexpr int NB = V / 4;
+  Polar2 pp[NB];
+  polar_blocks<NoiseForm::kScalar, NB>(gen, j0, pp);
 #pragma unroll
-  for (int b = 0; b < V / 4; ++b) {
-    const uint4 x = gen.block(j0 + b);
-    const Polar p = polar(x.x, x.y);
-    const Polar q = polar(x.z, x.w);
+  for (int b = 0; b < NB; ++b) {
+    const Polar2& p = pp[b];
     float h[4];
-    h[0] = fmaf(-(s1 * p.r), p.c, f[4 * b + 0]);
-    h[1] = fmaf(-(s1 * p.r), p.s, f[4 * b + 1]);
-    h[2] = fmaf(-(s1 * q.r), q.c, f[4 * b + 2]);
-    h[3] = fmaf(-(s1 * q.r), q.s, f[4 * b + 3]);
+    h[0] = fmaf(-(s1 * p.r.x), p.c.x, f[4 * b + 0]);
+    h[1] = fmaf(-(s1 * p.r.x), p.s.x, f[4 * b + 1]);
+    h[2] = fmaf(-(s1 * p.r.y), p.c.y, f[4 * b + 2]);
+    h[3] = fmaf(-(s1 * p.r.y), p.s.y, f[4 * b + 3]);
     Io::round_trip(h);
-    f[4 * b + 0] = fmaf(-(s2 * p.r), p.c, h[0]);
-    f[4 * b + 1] = fmaf(-(s2 * p.r), p.s, h[1]);
-    f[4 * b + 2] = fmaf(-(s2 * q.r), q.c, h[2]);
-    f[4 * b + 3] = fmaf(-(s2 * q.r), q.s, h[3]);
+    f[4 * b + 0] = fmaf(-(s2 * p.r.x), p.c.x, h[0]);
+    f[4 * b + 1] = fmaf(-(s2 * p.r.x), p.s.x, h[1]);
+    f[4 * b + 2] = fmaf(-(s2 * p.r.y), p.c.y, h[2]);
+    f[4 * b + 3] = fmaf(-(s2 * p.r.y), p.s.y, h[3]);
   }
 }
 

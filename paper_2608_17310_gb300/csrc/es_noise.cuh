@@ -221,15 +221,26 @@ __device__ __forceinline__ void sincos_approx(float a, float* s, float* c) {
 }
 
 // radius^2 = -2 ln u for u = uniform_open(x), fast path:
-//   for u <= 1 - 2^-10: -2 ln 2 * log2(u) with the MUFU log2 (log2_approx);
+//   for u <= 1 - 2^-10: -2 ln 2 * log2(u) with the MUFU log2 (radius_sq_log);
 //   for u >  1 - 2^-10: 2t + t^2 with t = 1 - u (exact); the dropped terms
-//     (2/3 t^3 + ...) are below t^2/3 <= 3.2e-7 relative.
-// Both are evaluated and one is selected, which keeps the code free of
-// divergent branches.
-__device__ __forceinline__ float radius_sq(float u) {
+//     (2/3 t^3 + ...) are below t^2/3 <= 3.2e-7 relative (radius_sq_series).
+// radius_sq evaluates both and selects one, which keeps the code free of
+// divergent branches. Since u = (2m + 1) 2^-24 with m = x >> 9, u > 1 - 2^-10
+// exactly when m >= 2^23 - 2^13, i.e. when the raw word x >= kNearOneWord; the
+// streaming kernels test that instead and compute the series only on a rare
+// branch (one radius input in 1024), with the same values.
+constexpr uint32_t kNearOneWord = 0xFFC00000u;
+
+__device__ __forceinline__ float radius_sq_log(float u) { return log2_approx(u) * kMinusTwoLn2; }
+
+__device__ __forceinline__ float radius_sq_series(float u) {
   const float t = 1.0f - u;
-  const float series = fmaf(t, t, t + t);
-  const float logged = log2_approx(u) * kMinusTwoLn2;
+  return fmaf(t, t, t + t);
+}
+
+__device__ __forceinline__ float radius_sq(float u) {
+  const float series = radius_sq_series(u);
+  const float logged = radius_sq_log(u);
   return u > kNearOne ? series : logged;
 }
 
@@ -249,11 +260,22 @@ struct Polar {
   float r, c, s;
 };
 
-__device__ __forceinline__ Polar polar(uint32_t xa, uint32_t xb) {
+// The pair before the square root: .r holds radius^2, from radius_sq (kLogOnly
+// false) or from the hardware log2 alone (kLogOnly true; the caller then
+// replaces the near-one inputs' radius^2 by radius_sq_series).
+template <bool kLogOnly>
+__device__ __forceinline__ Polar polar_sq(uint32_t xa, uint32_t xb) {
   Polar p;
-  p.r = sqrt_approx(radius_sq(uniform_open(xa)));
+  const float u = uniform_open(xa);
+  p.r = kLogOnly ? radius_sq_log(u) : radius_sq(u);
   const float f = one_plus_top23(xb);
   sincos_approx(fmaf(f, kTwoPi, kAngleOffset), &p.s, &p.c);
+  return p;
+}
+
+__device__ __forceinline__ Polar polar(uint32_t xa, uint32_t xb) {
+  Polar p = polar_sq<false>(xa, xb);
+  p.r = sqrt_approx(p.r);
   return p;
 }
 
@@ -267,23 +289,35 @@ struct Polar2 {
   float2 r, c, s;
 };
 
-__device__ __forceinline__ Polar2 polar2(const uint4& x) {
+// Both pairs before their square roots (.r holds radius^2), as polar_sq.
+template <bool kLogOnly>
+__device__ __forceinline__ Polar2 polar2_sq(const uint4& x) {
   Polar2 p;
   const float2 fa = make_float2(one_plus_top23(x.x), one_plus_top23(x.z));
   const float kHalfUlpBelowOne = __uint_as_float(0x3F7FFFFFu);
   const float2 u = __fadd2_rn(fa, make_float2(-kHalfUlpBelowOne, -kHalfUlpBelowOne));
-  const float2 t = __fadd2_rn(make_float2(1.0f, 1.0f), make_float2(-u.x, -u.y));
-  const float2 series = __ffma2_rn(t, t, __fadd2_rn(t, t));
   const float2 logged =
       __fmul2_rn(make_float2(log2_approx(u.x), log2_approx(u.y)),
                  make_float2(kMinusTwoLn2, kMinusTwoLn2));
-  p.r.x = sqrt_approx(u.x > kNearOne ? series.x : logged.x);
-  p.r.y = sqrt_approx(u.y > kNearOne ? series.y : logged.y);
+  if constexpr (kLogOnly) {
+    p.r = logged;
+  } else {
+    const float2 t = __fadd2_rn(make_float2(1.0f, 1.0f), make_float2(-u.x, -u.y));
+    const float2 series = __ffma2_rn(t, t, __fadd2_rn(t, t));
+    p.r.x = u.x > kNearOne ? series.x : logged.x;
+    p.r.y = u.y > kNearOne ? series.y : logged.y;
+  }
   const float2 fb = make_float2(one_plus_top23(x.y), one_plus_top23(x.w));
   const float2 ang = __ffma2_rn(fb, make_float2(kTwoPi, kTwoPi),
                                 make_float2(kAngleOffset, kAngleOffset));
   sincos_approx(ang.x, &p.s.x, &p.c.x);
   sincos_approx(ang.y, &p.s.y, &p.c.y);
+  return p;
+}
+
+__device__ __forceinline__ Polar2 polar2(const uint4& x) {
+  Polar2 p = polar2_sq<false>(x);
+  p.r = make_float2(sqrt_approx(p.r.x), sqrt_approx(p.r.y));
   return p;
 }
 

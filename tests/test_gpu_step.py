@@ -745,3 +745,78 @@ def test_two_plans_on_two_streams_equal_the_sequential_result(es):
         assert torch.equal(_int_view(x), _int_view(y))
     for p in plans:
         p.close()
+
+
+def _near_one_elements(oracle, seed, nblocks, threshold):
+    """Elements (ascending) of the Box-Muller pairs whose radius word is at least
+    `threshold`, within Philox blocks 0 .. nblocks - 1 of `seed` (the oracle's
+    words)."""
+    w = oracle.noise_blocks(seed, 0, nblocks)
+    b0 = np.nonzero(w[:, 0] >= threshold)[0].astype(np.uint64)
+    b2 = np.nonzero(w[:, 2] >= threshold)[0].astype(np.uint64)
+    return np.unique(np.concatenate([4 * b0, 4 * b0 + 1, 4 * b2 + 2, 4 * b2 + 3]))
+
+
+@pytest.mark.parametrize("dtype", ["f32", "bf16"])
+def test_near_one_radius_inputs_match_oracle(es, oracle, dtype):
+    # Radius inputs within 2^-10 of 1 (raw word >= 0xFFC00000, one pair in
+    # 1024) take the series of -2 ln u on a branch of their own in every
+    # kernel. From theta = 0 each call's output is its rounded noise term, so
+    # these elements are compared with the oracle directly: all near-one pairs
+    # of 2^21 blocks per seed, and in particular those within 2^-20 of 1
+    # (word >= 0xFFFFF000), where the hardware log2 alone would miss the
+    # tolerance several times over.
+    nblocks = 1 << 21
+    n = 4 * nblocks
+    tdt = torch.bfloat16 if dtype == "bf16" else torch.float32
+    theta = torch.zeros(n, dtype=tdt, device="cuda")
+    plan, segs = build_plan(es, [theta], [0])
+    seeds = [3, 2**33 + 9, 77, 2**60 + 1, 12345, 2**40 + 5]
+    near = {s: _near_one_elements(oracle, s, nblocks, 0xFFC00000) for s in seeds}
+    sharp = sum(_near_one_elements(oracle, s, nblocks, 0xFFFFF000).size for s in seeds)
+    assert sharp >= 8 and all(v.size > 6000 for v in near.values())
+    zeros = lambda m: np.zeros(m, dtype=np.uint16 if dtype == "bf16" else np.float32)
+    sigma = 1e-3
+
+    def gather(sel):
+        return host_values(theta[torch.from_numpy(sel.astype(np.int64)).cuda()])
+
+    for k, s in enumerate(seeds):
+        sel = near[s]
+        eps = oracle.noise_at(s, sel)
+        # one-seed pass
+        theta.zero_()
+        es.es_perturb(plan, s, sigma)
+        torch.cuda.synchronize()
+        compare(dtype, gather(sel), oracle.perturb(zeros(sel.size), sel, s, sigma, dtype),
+                f"es_perturb, seed {s}", noise_abs_tol([eps], [sigma]))
+        # two-seed pass: restore of s, perturb of the next seed (its near-one
+        # elements too)
+        s2 = seeds[(k + 1) % len(seeds)]
+        sel2 = np.union1d(sel, near[s2])
+        theta.zero_()
+        es.es_restore_perturb(plan, s, sigma, s2, sigma)
+        torch.cuda.synchronize()
+        mid = oracle.restore(zeros(sel2.size), sel2, s, sigma, dtype)
+        compare(dtype, gather(sel2), oracle.perturb(mid, sel2, s2, sigma, dtype),
+                f"es_restore_perturb, seeds {s}, {s2}",
+                noise_abs_tol([oracle.noise_at(s, sel2), oracle.noise_at(s2, sel2)],
+                              [sigma, sigma]))
+        # update over two seeds, then the fused update + next perturb
+        coeffs = np.array([2.5e-4, -1.5e-4], dtype=np.float32)
+        theta.zero_()
+        es.es_update(plan, np.array([s, s2], dtype=np.uint64), coeffs)
+        torch.cuda.synchronize()
+        tol = noise_abs_tol([oracle.noise_at(s, sel2), oracle.noise_at(s2, sel2)], coeffs)
+        compare(dtype, gather(sel2),
+                oracle.update(zeros(sel2.size), sel2, [s, s2], coeffs, dtype),
+                f"es_update, seeds {s}, {s2}", tol)
+        theta.zero_()
+        es.es_update_perturb(plan, np.array([s2], dtype=np.uint64), coeffs[:1], s, sigma)
+        torch.cuda.synchronize()
+        upd = oracle.update(zeros(sel2.size), sel2, [s2], coeffs[:1], dtype)
+        compare(dtype, gather(sel2), oracle.perturb(upd, sel2, s, sigma, dtype),
+                f"es_update_perturb, seeds {s2} then {s}",
+                noise_abs_tol([oracle.noise_at(s2, sel2), oracle.noise_at(s, sel2)],
+                              [coeffs[0], sigma]))
+    plan.close()

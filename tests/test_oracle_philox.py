@@ -94,3 +94,12 @@ def test_philox_output_bits_are_uniform(oracle):
     ones = bits.sum(axis=0)
     assert np.all(np.abs(ones - n / 2) < 6 * np.sqrt(n) / 2)
     assert len(np.unique(words.ravel())) > 4 * n - 10
+
+
+def test_noise_blocks_is_noise_block_over_a_range(oracle):
+    # the bulk form (used to find inputs with given raw words) gives each
+    # block's words, across the 2^32-block boundary of the counter's low word
+    for seed, j0 in ((5, 0), (2**40 + 3, 2**32 - 3)):
+        w = oracle.noise_blocks(seed, j0, 7)
+        for k in range(7):
+            assert np.array_equal(w[k], oracle.noise_block(seed, j0 + k))
