@@ -221,26 +221,6 @@ constexpr NoiseForm kUpdateForm = static_cast<NoiseForm>(ES_UPDATE_FORM);
 // Near-one radius inputs: a rare branch (true) or a select per pair (false).
 constexpr bool kNearOneBranch = ES_NEAR_ONE_BRANCH != 0;
 
-// Radius^2 of every pair of NB Philox blocks (p[b].r, from the hardware log2)
-// corrected where the radius input lies within 2^-10 of 1: such a pair takes
-// the series instead. The test is on the raw words (xa[b] = the blocks' words
-// x0 and x2), and the series is computed only when some pair needs it (one
-// radius input in 1024), so the common path costs one compare per pair. The
-// values equal radius_sq's.
-template <int NB>
-__device__ __forceinline__ void fix_near_one(const uint2 (&xa)[NB], Polar2 (&p)[NB]) {
-  bool near = false;
-#pragma unroll
-  for (int b = 0; b < NB; ++b) near |= (xa[b].x >= kNearOneWord) | (xa[b].y >= kNearOneWord);
-  if (__builtin_expect(near, 0)) {
-#pragma unroll
-    for (int b = 0; b < NB; ++b) {
-      if (xa[b].x >= kNearOneWord) p[b].r.x = radius_sq_series(uniform_open(xa[b].x));
-      if (xa[b].y >= kNearOneWord) p[b].r.y = radius_sq_series(uniform_open(xa[b].y));
-    }
-  }
-}
-
 // The pairs of Philox blocks j0 .. j0 + NB - 1 in polar form (r, cos, sin),
 // .x of each Polar2 the block's pair (x0, x1), .y its pair (x2, x3).
 template <NoiseForm kForm, int NB, class Gen>

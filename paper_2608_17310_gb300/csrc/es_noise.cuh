@@ -321,6 +321,26 @@ __device__ __forceinline__ Polar2 polar2(const uint4& x) {
   return p;
 }
 
+// Radius^2 of every pair of NB Philox blocks (p[b].r, from the hardware log2)
+// corrected where the radius input lies within 2^-10 of 1: such a pair takes
+// the series instead. The test is on the raw words (xa[b] = the blocks' words
+// x0 and x2), and the series is computed only when some pair needs it (one
+// radius input in 1024), so the common path costs one compare per pair. The
+// values equal radius_sq's.
+template <int NB>
+__device__ __forceinline__ void fix_near_one(const uint2 (&xa)[NB], Polar2 (&p)[NB]) {
+  bool near = false;
+#pragma unroll
+  for (int b = 0; b < NB; ++b) near |= (xa[b].x >= kNearOneWord) | (xa[b].y >= kNearOneWord);
+  if (__builtin_expect(near, 0)) {
+#pragma unroll
+    for (int b = 0; b < NB; ++b) {
+      if (xa[b].x >= kNearOneWord) p[b].r.x = radius_sq_series(uniform_open(xa[b].x));
+      if (xa[b].y >= kNearOneWord) p[b].r.y = radius_sq_series(uniform_open(xa[b].y));
+    }
+  }
+}
+
 // One Box-Muller pair, materialised.
 __device__ __forceinline__ float2 box_muller(uint32_t xa, uint32_t xb) {
   const Polar p = polar(xa, xb);

@@ -22,7 +22,9 @@
 //                  (or only one half runs): whether the two pipes overlap at
 //                  all when their instructions come from different warps;
 //   generator      the library's own Philox4x32-10 (es_noise.cuh) in blocks,
-//                  and the full generator (Philox + Box-Muller) in Gaussians.
+//                  and the full generator in Gaussians in the form the
+//                  streaming kernels use (scheduled round keys, packed
+//                  transform, near-one series on a rare branch).
 #include <cuda_runtime.h>
 
 #include <cstdint>
@@ -277,16 +279,29 @@ probe_kernel(int iters, uint32_t seed, unsigned long long* __restrict__ rec,
       j += 0x20000u;
     }
   } else if constexpr (P == kGenerator) {
-    const esopt::PhiloxTile pt = esopt::philox_tile(0u, esopt::philox_key(seed));
+    // the kernels' generator: round keys from a precomputed schedule, the
+    // packed transform from the hardware log2, the near-one series on a rare
+    // branch, then the square roots
+    const esopt::PhiloxSched ps = esopt::philox_sched(seed);
+    const esopt::TileConst tc = esopt::tile_const(0u, ps.rk[0], ps.rk[3]);
     uint32_t j = t * 2u;
     float2 s0 = make_float2(0.f, 0.f), s1 = s0;
 #pragma unroll 1
     for (int i = 0; i < iters; ++i) {
+      uint2 xa[2];
+      esopt::Polar2 p[2];
 #pragma unroll
       for (int b = 0; b < 2; ++b) {
-        const esopt::Polar2 p = esopt::polar2(esopt::philox_block_tile(j + b, pt));
-        s0 = __ffma2_rn(make_float2(p.r.x, p.r.x), make_float2(p.c.x, p.s.x), s0);
-        s1 = __ffma2_rn(make_float2(p.r.y, p.r.y), make_float2(p.c.y, p.s.y), s1);
+        const uint4 x = esopt::philox_block_rk(j + b, tc, ps.rk[1], ps.rk[2], ps.rk + 4);
+        xa[b] = make_uint2(x.x, x.z);
+        p[b] = esopt::polar2_sq<true>(x);
+      }
+      esopt::fix_near_one<2>(xa, p);
+#pragma unroll
+      for (int b = 0; b < 2; ++b) {
+        const float2 r = make_float2(esopt::sqrt_approx(p[b].r.x), esopt::sqrt_approx(p[b].r.y));
+        s0 = __ffma2_rn(make_float2(r.x, r.x), make_float2(p[b].c.x, p[b].s.x), s0);
+        s1 = __ffma2_rn(make_float2(r.y, r.y), make_float2(p[b].c.y, p[b].s.y), s1);
       }
       j += 0x20000u;
     }
