@@ -1,8 +1,9 @@
 """The e2e leg of bench.py computes exactly the generation it times: its
 grouped schedule (copy in, first pass per group plan, middle passes on the
-whole plan, last pass per group plan, copy out) leaves, after two generations,
-the host buffer and the device buffer bit-identical to the whole-plan loop
-that the device-timed leg runs."""
+whole plan, last pass per group plan, copy out, and with pipelining the next
+step's copy in right after each group's copy out) leaves, after three
+generations, the host buffer and the device buffer bit-identical to the
+whole-plan loop that the device-timed leg runs."""
 import numpy as np
 import pytest
 import torch
@@ -12,8 +13,10 @@ from paper_2608_17310_gb300 import inputs as I
 pytestmark = pytest.mark.gpu
 
 
-@pytest.mark.parametrize("fused,population", [(True, None), (False, None), (True, 1)])
-def test_e2e_leg_equals_the_device_loop(es, fused, population):
+@pytest.mark.parametrize("fused,population,pipelined",
+                         [(True, None, True), (True, None, False), (False, None, True),
+                          (True, 1, True)])
+def test_e2e_leg_equals_the_device_loop(es, fused, population, pipelined):
     import bench
     name = "qwen4b_4layer"
     wl = I.WORKLOADS[name]
@@ -34,8 +37,9 @@ def test_e2e_leg_equals_the_device_loop(es, fused, population):
     bench.start_loop(es, plan, wl, 0, n, sigma_at(0), sh, fused)
     bench.start_loop(es, twin_plan, wl, 0, n, sigma_at(0), sh, fused)
     loop = bench.E2ELoop(torch, es, plan, flat, params, wl, n, 2, sigma_at, sh, fused)
-    for t in range(2):
-        loop.step(t)
+    for t in range(3):
+        # pipelined: each step issues the next step's copies to the device
+        loop.step(t, copy_next=pipelined and t < 2)
         bench.run_step(es, twin_plan, wl, t, n, sigma_at(t), sigma_at(t + 1), sh, None, fused)
     torch.cuda.synchronize()
     want = twin_flat.view(torch.int16)
