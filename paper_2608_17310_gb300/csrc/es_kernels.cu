@@ -179,13 +179,13 @@ struct TileGen {
   PhiloxTile t;
   __device__ uint4 block(uint64_t j) const { return philox_block_tile(static_cast<uint32_t>(j), t); }
 };
-template <class Keys>
+template <class Keys, bool kWideFirst = false>
 struct SchedGen {
   TileConst t;
   uint32_t rk1, rk2;  // round 0's k1, round 1's k0
   Keys rk;            // rounds 2..9: rk[2r - 4], rk[2r - 3]
   __device__ uint4 block(uint64_t j) const {
-    return philox_block_rk(static_cast<uint32_t>(j), t, rk1, rk2, rk);
+    return philox_block_rk<kWideFirst>(static_cast<uint32_t>(j), t, rk1, rk2, rk);
   }
 };
 struct AnyGen {
@@ -200,10 +200,11 @@ __device__ __forceinline__ auto make_gen(PhiloxKey key, uint32_t j_hi) {
 }
 
 // Generator of one seed whose schedule is a kernel parameter.
-template <bool kUniformHi>
+template <bool kUniformHi, bool kWideFirst = false>
 __device__ __forceinline__ auto sched_gen(const PhiloxSched& s, uint32_t j_hi) {
   if constexpr (kUniformHi)
-    return SchedGen<const uint32_t*>{tile_const(j_hi, s.rk[0], s.rk[3]), s.rk[1], s.rk[2], s.rk + 4};
+    return SchedGen<const uint32_t*, kWideFirst>{tile_const(j_hi, s.rk[0], s.rk[3]), s.rk[1],
+                                                 s.rk[2], s.rk + 4};
   else return AnyGen{PhiloxKey{s.rk[0], s.rk[1]}};
 }
 
@@ -392,7 +393,8 @@ __device__ __forceinline__ void axpy_tile(const TileRef<Io>& cur, uint4 (&v)[G],
   constexpr int kGroups = kVecsPerThread / G;
   constexpr int kStride = kBlockThreads * V;  // elements from one vector of a thread to the next
   const uint32_t j_hi = static_cast<uint32_t>((cur.index_base + cur.t0) >> 34);
-  const auto gen = sched_gen<kUniformHi>(a.s1, j_hi);
+  // the one-seed pass is fastest with every Philox product 64-bit wide
+  const auto gen = sched_gen<kUniformHi, !kTwo>(a.s1, j_hi);
   const auto gen2 = sched_gen<kUniformHi && kTwo && !kSame>(a.s2, j_hi);
   const float s1 = a.scale1 * cur.inv, s2 = a.scale2 * cur.inv;
   // the thread's first element of the tile, and its Philox block (index_base

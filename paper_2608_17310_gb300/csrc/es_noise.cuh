@@ -150,14 +150,26 @@ __device__ __forceinline__ TileConst tile_const(uint32_t j_hi, uint32_t k0, uint
 
 // philox_block_tile with the round keys taken from a schedule: `rk1` is round
 // 0's k1, `rk2` round 1's k0, `rk` points at the keys of rounds 2..9 (rk[2r - 4],
-// rk[2r - 3] for round r). Bit-identical to philox_block.
-template <class Keys>
+// rk[2r - 3] for round r). kWideFirst: the first two rounds' products also as
+// one 64-bit-result multiply each (a high/low pair costs the integer pipe more
+// cycles, but one more instruction issue less; which is faster depends on the
+// kernel). Bit-identical to philox_block.
+template <bool kWideFirst, class Keys>
 __device__ __forceinline__ uint4 philox_block_rk(uint32_t j_lo, TileConst t, uint32_t rk1,
                                                  uint32_t rk2, const Keys& rk) {
-  const uint32_t a2 = mul_hi(kPhiloxMulA, j_lo) ^ rk1;  // round 0, word 2
-  const uint32_t a3 = mul_lo(kPhiloxMulA, j_lo);        // round 0, word 3
-  uint32_t c0 = mul_hi(kPhiloxMulB, a2) ^ rk2;          // round 1 (its word 1 was 0)
-  uint32_t c1 = mul_lo(kPhiloxMulB, a2);
+  uint32_t a2, a3, c0, c1;
+  if constexpr (kWideFirst) {
+    uint32_t h0, h1;
+    mul_wide(kPhiloxMulA, j_lo, h0, a3);  // round 0: words 2 and 3
+    a2 = h0 ^ rk1;
+    mul_wide(kPhiloxMulB, a2, h1, c1);    // round 1 (its word 1 was 0)
+    c0 = h1 ^ rk2;
+  } else {
+    a2 = mul_hi(kPhiloxMulA, j_lo) ^ rk1;  // round 0, word 2
+    a3 = mul_lo(kPhiloxMulA, j_lo);        // round 0, word 3
+    c0 = mul_hi(kPhiloxMulB, a2) ^ rk2;    // round 1 (its word 1 was 0)
+    c1 = mul_lo(kPhiloxMulB, a2);
+  }
   uint32_t c2 = t.x2 ^ a3;
   uint32_t c3 = t.lo2;
 #pragma unroll

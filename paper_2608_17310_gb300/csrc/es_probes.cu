@@ -292,7 +292,7 @@ probe_kernel(int iters, uint32_t seed, unsigned long long* __restrict__ rec,
       esopt::Polar2 p[2];
 #pragma unroll
       for (int b = 0; b < 2; ++b) {
-        const uint4 x = esopt::philox_block_rk(j + b, tc, ps.rk[1], ps.rk[2], ps.rk + 4);
+        const uint4 x = esopt::philox_block_rk<false>(j + b, tc, ps.rk[1], ps.rk[2], ps.rk + 4);
         xa[b] = make_uint2(x.x, x.z);
         p[b] = esopt::polar2_sq<true>(x);
       }
