@@ -78,6 +78,9 @@ def parse():
                    help="instead of the step: the register-only pipe probes (integer "
                         "multiply, MUFU, FMA, LOP3, their mixes, a warp-split overlap test, "
                         "the generator) in ops per clock per SM")
+    p.add_argument("--probes", default=None,
+                   help="--pipe-peaks: only these probes (comma-separated names), at 4 CTAs "
+                        "per SM")
     p.add_argument("--antithetic", action="store_true",
                    help="instead of the step: a generation of N/2 antithetic pairs (the +/- "
                         "flip as one es_restore_perturb on one seed)")
@@ -468,7 +471,7 @@ def run_ours(args, rank, world, dist):
     per_step_ms = ms_max / args.steps
     value = world * P * n * args.steps / (ms_max / 1e3)
 
-    imul_peak, gauss_peak, measured_peak, sms, sm_max_mhz, hbm_gbs, peak_src, ceilings = \
+    imul_peak, gauss_peak, gen_peak, sms, sm_max_mhz, hbm_gbs, peak_src, ceilings = \
         alu_peaks(torch, dev_index)
     bytes_per_launch = 2 * esize * P
     kernels = {}
@@ -481,7 +484,7 @@ def run_ours(args, rank, world, dist):
         kernels[name] = {"kernel": KERNEL_NAME[name], "launches": timers.count(name),
                          "mean_ms": mean, "share": timers.total_ms(name) / ms,
                          "gbs": gbs, "gauss_per_s": gps, "hbm_frac": hbm_frac,
-                         "alu_frac": alu_frac, "measured_alu_frac": gps / measured_peak,
+                         "alu_frac": alu_frac, "generator_frac": gps / gen_peak,
                          "bound": "alu" if alu_frac > hbm_frac else "hbm"}
     dom = max(kernels, key=lambda k: kernels[k]["share"])
     d = kernels[dom]
@@ -497,13 +500,12 @@ def run_ours(args, rank, world, dist):
                 "traffic": traffic,
                 "peak_source": f"{sms} SMs x {IMUL_PER_CLK_SM} 32-bit integer multiplies/clk x "
                                f"{sm_max_mhz:.0f} MHz; {IMUL_PER_GAUSS} multiplies per Gaussian"}
-    roof["measured_alu_bound"] = {
-        "gauss_per_s": measured_peak, "frac": d["gauss_per_s"] / measured_peak,
-        "binding_pipe": ceilings["alu"]["binding_pipe"],
-        "source": "measured in this run: the method's mandated ALU work per Gaussian (4.5 "
-                  "mad.wide.u32, 4.75 lop3, 2 MUFU) over each pipe's rate in register-only "
-                  "probes at 4 CTAs per SM, the slowest pipe binding, scaled to the maximum SM "
-                  "clock (bench.py --pipe-peaks has every probe)"}
+    roof["generator_bound"] = {
+        "gauss_per_s": gen_peak, "frac": d["gauss_per_s"] / gen_peak,
+        "source": "measured in this run: the kernels' own generator (Philox, Box-Muller) in a "
+                  "register-only loop with no memory traffic, 4 CTAs per SM, scaled to the "
+                  "maximum SM clock: what this instruction stream reaches on its own "
+                  "(bench.py --pipe-peaks has every probe)"}
     roof["measured_ceilings"] = ceilings
     roof["pipe_occupancy"] = pipe_occupancy(dom)
     roof.update({"kernel": d["kernel"], "hbm_frac": d["hbm_frac"], "alu_frac": d["alu_frac"],
@@ -579,30 +581,29 @@ def run_probe(L, name, ctas_per_sm=4, target_ms=20.0):
 def measured_ceilings(res, sms, sm_max_mhz):
     """ALU ceilings of the generator from probe results (`res`: name -> run_probe
     dict), in Gaussians/s at the maximum SM clock:
-      imad_wide      the integer-multiply pipe alone: mad.wide.u32 rate / 4.5;
+      imad_wide      a chain of mad.wide.u32 with a 64-bit addend, per 4.5 per
+                     Gaussian. ncu counts 1.5 FMA-heavy instructions and 5 pipe
+                     cycles per operation of this chain, against 4 cycles for
+                     the kernels' mul.wide, so it understates the pipe: the
+                     nominal 64 multiplies per clock per SM (32 mul.wide at 4
+                     cycles each) is the pipe's rate;
       lop3           the three-input XOR alone: lop3 rate / 4.75;
       mufu           the MUFU pipe alone: its rate / 2;
-      alu            the bound of the method's mandated ALU work with these
-                     measured pipe peaks: t_ALU per Gaussian = the maximum over
-                     the three pipes of mandated ops / measured rate;
       imad_mufu_mix  mad.wide and MUFU in the generator's ratio (9 : 4) in one
                      thread;
-      generator      the library's full generator (Philox + Box-Muller) in
-                     registers, no memory traffic."""
+      generator      the streaming kernels' generator (Philox with scheduled
+                     round keys, the packed transform, the near-one series on a
+                     rare branch) in registers, no memory traffic: the rate this
+                     instruction stream reaches on its own."""
     hz = sms * sm_max_mhz * 1e6
     out = {}
-    per_pipe = {}
     for name, per_g in (("imad_wide", WIDE_PER_GAUSS), ("lop3", LOP3_PER_GAUSS),
                         ("mufu", MUFU_PER_GAUSS)):
         if name in res:
             r = res[name]["ops_per_clk_sm"]
             out[name] = {"ops_per_clk_sm": r, "per_gaussian": per_g, "gauss_per_s": r / per_g * hz}
-            per_pipe[name] = r / per_g * hz
     if "imad_wide" in out:
         out["imad_wide"]["imul32_per_clk_sm"] = 2 * out["imad_wide"]["ops_per_clk_sm"]
-    if per_pipe:
-        pipe = min(per_pipe, key=per_pipe.get)
-        out["alu"] = {"gauss_per_s": per_pipe[pipe], "binding_pipe": pipe}
     if "mix_imad_wide_mufu_9_4" in res:
         r = res["mix_imad_wide_mufu_9_4"]["ops_per_clk_sm"]
         out["imad_mufu_mix"] = {"wide_per_clk_sm": r, "gauss_per_s": r / WIDE_PER_GAUSS * hz}
@@ -631,19 +632,19 @@ CEILING_PROBES = ("imad_wide", "lop3", "mufu", "mix_imad_wide_mufu_9_4", "mix_im
 
 def alu_peaks(torch, dev_index, probes=True):
     """(imul32/s at the nominal integer-multiply rate, Gaussians/s at that
-    roofline, Gaussians/s at the measured ALU bound, SM count, max SM MHz, HBM
-    GB/s, peak source, measured ceilings).
+    roofline, Gaussians/s of the register-only generator, SM count, max SM MHz,
+    HBM GB/s, peak source, measured ceilings).
 
     The roofline is the nominal one: 64 32-bit multiplies per clock per SM x
-    SMs x the maximum SM clock, 9 multiplies per Gaussian. The measured ALU
-    bound takes the same mandated work against the pipe peaks that the
-    register-only probes measure live (mad.wide.u32, lop3, MUFU; the slowest
-    pipe binds); without probes it is None."""
+    SMs x the maximum SM clock, 9 multiplies per Gaussian. It is the FMA-heavy
+    pipe's rate for mul.wide.u32 (4 pipe cycles per warp instruction, ncu). The
+    generator rate is measured live by the register-only probe of the kernels'
+    own generator (no memory traffic); without probes it is None."""
     hbm_gbs, sm_max_mhz, peak_src = peaks()
     sms = torch.cuda.get_device_properties(dev_index).multi_processor_count
     imul_peak = sms * IMUL_PER_CLK_SM * sm_max_mhz * 1e6
     ceilings = {}
-    measured_peak = None
+    gen_peak = None
     if probes:
         L = probe_lib()
         res = {name: run_probe(L, name, 4, 10.0) for name in CEILING_PROBES}
@@ -652,8 +653,8 @@ def alu_peaks(torch, dev_index, probes=True):
                               "of 256 threads per SM, each SM timed on its own clock from its "
                               "first CTA's start to its last CTA's end, scaled to the maximum "
                               "SM clock")
-        measured_peak = ceilings["alu"]["gauss_per_s"]
-    return (imul_peak, imul_peak / IMUL_PER_GAUSS, measured_peak, sms, sm_max_mhz, hbm_gbs,
+        gen_peak = ceilings["generator"]["gauss_per_s"]
+    return (imul_peak, imul_peak / IMUL_PER_GAUSS, gen_peak, sms, sm_max_mhz, hbm_gbs,
             peak_src, ceilings)
 
 
@@ -670,12 +671,20 @@ def run_pipe_peaks(args, rank, world, dist):
     sms = torch.cuda.get_device_properties(dev_index).multi_processor_count
     L = probe_lib()
     names = [L.esprobe_name(i).decode() for i in range(L.esprobe_count())]
+    if args.probes:
+        wanted = [x.strip() for x in args.probes.split(",") if x.strip()]
+        unknown = [x for x in wanted if x not in names]
+        if unknown:
+            raise SystemExit(f"--probes: unknown probe(s) {unknown}; known: {names}")
+        names = wanted
     res, occupancy = {}, []
     with ClockSampler(dev_index) as clk:
         for name in names:
             res[name] = run_probe(L, name, 4, 25.0)
         for name in ("imad_wide", "mufu", "mix_imad_wide_mufu_9_4", "mix_imad_hi_lo_1_1",
                      "mix_imad_hi_lo_mufu_9_4", "philox", "generator"):
+            if args.probes:
+                break
             for ctas in (1, 2, 8):
                 occupancy.append(run_probe(L, name, ctas, 25.0))
     out = {"mode": "pipe_peaks", "metric": "ops per clock per SM of register-only pipe probes",
@@ -707,7 +716,7 @@ def run_sweep(args, rank, world, dist):
     P = plan.numel
     stream = torch.cuda.current_stream()
     s_handle = stream.cuda_stream
-    imul_peak, gauss_peak, measured_peak, sms, sm_max_mhz, hbm_gbs, peak_src, _ = \
+    imul_peak, gauss_peak, gen_peak, sms, sm_max_mhz, hbm_gbs, peak_src, _ = \
         alu_peaks(torch, dev_index)
     bytes_per_launch = 2 * esize * P
     pops = [int(x) for x in args.populations.split(",") if x.strip()]
@@ -739,15 +748,14 @@ def run_sweep(args, rank, world, dist):
             gps = n * P / (ms / 1e3)
             t_hbm = bytes_per_launch / (hbm_gbs * 1e9) * 1e3
             t_imul = n * P / gauss_peak * 1e3
-            t_measured = n * P / measured_peak * 1e3
+            t_gen = n * P / gen_peak * 1e3
             points.append({
                 "population": n, "mean_ms": ms, "gbs": gbs, "gauss_per_s": gps,
                 "hbm_frac": gbs / hbm_gbs, "alu_frac": gps / gauss_peak,
-                "measured_alu_frac": gps / measured_peak,
+                "generator_frac": gps / gen_peak,
                 "bound": "alu" if t_imul > t_hbm else "hbm",
                 "roofline_frac": max(t_hbm, t_imul) / ms,
-                "measured_roofline_frac": max(t_hbm, t_measured) / ms,
-                "t_hbm_ms": t_hbm, "t_imul_ms": t_imul, "t_alu_measured_ms": t_measured})
+                "t_hbm_ms": t_hbm, "t_imul_ms": t_imul, "t_generator_ms": t_gen})
     plan.close()
     out = {"mode": "sweep", "metric": "es_update param*seed/s per population size",
            "unit": UNIT, "n_gpus": 1, "steps": args.steps, "warmup": args.warmup,
@@ -757,7 +765,7 @@ def run_sweep(args, rank, world, dist):
                           rewards="N(0,1) used as the normalised rewards; paper-scale coefficients"),
            "peaks": {"hbm_gbs": hbm_gbs, "hbm_source": peak_src,
                      "imul32_per_s": imul_peak, "gauss_per_s_imul": gauss_peak,
-                     "gauss_per_s_alu_measured": measured_peak, "sms": sms,
+                     "gauss_per_s_generator": gen_peak, "sms": sms,
                      "sm_max_mhz": sm_max_mhz},
            "bytes_per_launch": bytes_per_launch, "points": points,
            "gpu_launches": launches, "clocks": clk.summary()}
@@ -779,11 +787,11 @@ def _timed(torch, stream, fn, reps):
 
 
 def _rates(P, gaussians_per_param, bytes_total, ms, peaks_):
-    imul_peak, gauss_peak, measured_peak, _, _, hbm_gbs, _, _ = peaks_
+    imul_peak, gauss_peak, gen_peak, _, _, hbm_gbs, _, _ = peaks_
     gps = gaussians_per_param * P / (ms / 1e3)
     gbs = bytes_total / (ms / 1e3) / 1e9
     return {"ms": ms, "gauss_per_s": gps, "gbs": gbs, "hbm_frac": gbs / hbm_gbs,
-            "alu_frac": gps / gauss_peak, "measured_alu_frac": gps / measured_peak}
+            "alu_frac": gps / gauss_peak, "generator_frac": gps / gen_peak}
 
 
 def run_replay(args, rank, world, dist):

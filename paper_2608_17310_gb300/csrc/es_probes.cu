@@ -55,6 +55,7 @@ enum Probe : int {
   kSplitBoth,
   kPhilox,
   kGenerator,
+  kImadWideMul,
   kProbeCount
 };
 
@@ -90,6 +91,7 @@ const ProbeInfo kInfo[kProbeCount] = {
     {"split_both", "warp-iterations (even warps mad.wide, odd warps MUFU)", 1, 1},
     {"philox", "Philox4x32-10 block", 2, 1},
     {"generator", "Gaussian (Philox4x32-10 + Box-Muller)", 8, 1},
+    {"imad_wide_mul", "mul.wide.u32 by a constant (no addend), with one add each", 8, 1},
 };
 
 __device__ __forceinline__ uint64_t mad_wide(uint32_t a, uint64_t c) {
@@ -278,6 +280,19 @@ probe_kernel(int iters, uint32_t seed, unsigned long long* __restrict__ rec,
       x[3] ^= a.w ^ b.w;
       j += 0x20000u;
     }
+  } else if constexpr (P == kImadWideMul) {
+    // Philox's form: the product by a constant without an addend; the high
+    // word feeds the chain, the low word an accumulator (one add on the ALU)
+#pragma unroll 1
+    for (int i = 0; i < iters; ++i)
+#pragma unroll
+      for (int k = 0; k < 8; ++k) {
+        uint32_t hi, lo;
+        asm volatile("{\n\t.reg .u64 p;\n\tmul.wide.u32 p, %2, %3;\n\tmov.b64 {%1, %0}, p;\n\t}"
+                     : "=r"(hi), "=r"(lo) : "r"(x[k]), "n"(kMul));
+        x[k] = hi;
+        y[k] += lo;
+      }
   } else if constexpr (P == kGenerator) {
     // the kernels' generator: round keys from a precomputed schedule, the
     // packed transform from the hardware log2, the near-one series on a rare
@@ -327,7 +342,7 @@ probe_kernel(int iters, uint32_t seed, unsigned long long* __restrict__ rec,
   for (int k = 0; k < 9; ++k) s ^= static_cast<uint32_t>(w[k] ^ (w[k] >> 32));
 #pragma unroll
   for (int k = 0; k < 8; ++k)
-    s ^= x[k] ^ __float_as_uint(f[k]) ^ __float_as_uint(f2[k].x) ^ __float_as_uint(f2[k].y);
+    s ^= x[k] ^ y[k] ^ __float_as_uint(f[k]) ^ __float_as_uint(f2[k].x) ^ __float_as_uint(f2[k].y);
 #pragma unroll
   for (int k = 0; k < 4; ++k) s ^= __float_as_uint(m[k]);
   if (s == seed * 0x2545F491u + 0x1234567u) sink[0] = s;
@@ -343,7 +358,7 @@ void* const kKernels[kProbeCount] = {
     kernel_of<4>(),  kernel_of<5>(),  kernel_of<6>(),  kernel_of<7>(),
     kernel_of<8>(),  kernel_of<9>(),  kernel_of<10>(), kernel_of<11>(),
     kernel_of<12>(), kernel_of<13>(), kernel_of<14>(), kernel_of<15>(),
-    kernel_of<16>(), kernel_of<17>(),
+    kernel_of<16>(), kernel_of<17>(), kernel_of<18>(),
 };
 
 }  // namespace
