@@ -699,18 +699,22 @@ noise_fill_kernel(uint64_t index_base, uint64_t n, PhiloxKey key, float* __restr
 // es_noise_fill when `out` is 16-byte aligned and index_base % 4 == 0:
 // out4[b] = eps[4 (j_first + b) .. 4 (j_first + b) + 3] for b < nblocks. Tiles
 // of 256 threads x kVecsPerThread blocks, each 16-byte store coalesced across
-// the warp; the Philox constants of the blocks' high word are hoisted per tile
-// when the tile stays within one 2^32-block range. The pair transform is the
-// packed form (bit-identical to box_muller).
+// the warp. The generator is the streaming kernels': round keys from the
+// launch's schedule, the Philox constants of the blocks' high word per tile
+// (when the tile stays within one 2^32-block range), the packed transform with
+// the near-one series on a rare branch (values equal to box_muller's).
 template <bool kUniformHi>
 __device__ __forceinline__ void noise_fill_tile(uint64_t j_first, uint64_t b0, uint64_t nblocks,
-                                                PhiloxKey key, float4* __restrict__ out) {
-  const auto gen = make_gen<kUniformHi>(key, static_cast<uint32_t>((j_first + b0) >> 32));
+                                                const PhiloxSched& sched,
+                                                float4* __restrict__ out) {
+  const auto gen = sched_gen<kUniformHi>(sched, static_cast<uint32_t>((j_first + b0) >> 32));
 #pragma unroll
   for (int q = 0; q < kVecsPerThread; ++q) {
     const uint64_t b = b0 + static_cast<uint64_t>(q * kBlockThreads + threadIdx.x);
     if (b < nblocks) {
-      const Polar2 p = polar2(gen.block(j_first + b));
+      Polar2 pp[1];
+      polar_blocks<NoiseForm::kPacked, 1>(gen, j_first + b, pp);
+      const Polar2& p = pp[0];
       const float2 lo = __fmul2_rn(make_float2(-p.r.x, -p.r.x), make_float2(p.c.x, p.s.x));
       const float2 hi = __fmul2_rn(make_float2(-p.r.y, -p.r.y), make_float2(p.c.y, p.s.y));
       out[b] = make_float4(lo.x, lo.y, hi.x, hi.y);
@@ -719,16 +723,17 @@ __device__ __forceinline__ void noise_fill_tile(uint64_t j_first, uint64_t b0, u
 }
 
 __global__ void __launch_bounds__(kBlockThreads)
-noise_fill_vec_kernel(uint64_t j_first, uint64_t nblocks, PhiloxKey key, float4* __restrict__ out) {
+noise_fill_vec_kernel(uint64_t j_first, uint64_t nblocks, const __grid_constant__ PhiloxSched sched,
+                      float4* __restrict__ out) {
   constexpr uint64_t kTileBlocks = static_cast<uint64_t>(kBlockThreads) * kVecsPerThread;
   const uint64_t tiles = (nblocks + kTileBlocks - 1) / kTileBlocks;
   for (uint64_t tile = blockIdx.x; tile < tiles; tile += gridDim.x) {
     const uint64_t b0 = tile * kTileBlocks;
     const uint64_t last = (b0 + kTileBlocks < nblocks ? b0 + kTileBlocks : nblocks) - 1;
     if (((j_first + b0) >> 32) == ((j_first + last) >> 32))
-      noise_fill_tile<true>(j_first, b0, nblocks, key, out);
+      noise_fill_tile<true>(j_first, b0, nblocks, sched, out);
     else
-      noise_fill_tile<false>(j_first, b0, nblocks, key, out);
+      noise_fill_tile<false>(j_first, b0, nblocks, sched, out);
   }
 }
 
@@ -877,7 +882,8 @@ cudaError_t launch_noise_fill(uint64_t seed, uint64_t index_base, uint64_t n, fl
     const uint64_t full = n / 4;
     constexpr uint64_t kTileBlocks = static_cast<uint64_t>(kBlockThreads) * kVecsPerThread;
     const int grid = persistent_grid(noise_fill_vec_kernel, (full + kTileBlocks - 1) / kTileBlocks);
-    noise_fill_vec_kernel<<<grid, kBlockThreads, 0, stream>>>(index_base / 4, full, key,
+    noise_fill_vec_kernel<<<grid, kBlockThreads, 0, stream>>>(index_base / 4, full,
+                                                              philox_sched(seed),
                                                               reinterpret_cast<float4*>(out));
     const cudaError_t err = cudaGetLastError();
     if (err != cudaSuccess || n % 4 == 0) return err;
