@@ -15,7 +15,10 @@ constexpr int kBlockThreads = 256;
 // 16-byte vectors per thread in one tile. A tile (kBlockThreads x
 // kVecsPerThread vectors) is the unit a CTA takes from a plan; tiles never
 // straddle segments.
-constexpr int kVecsPerThread = 4;
+#ifndef ES_VECS_PER_THREAD
+#define ES_VECS_PER_THREAD 4
+#endif
+constexpr int kVecsPerThread = ES_VECS_PER_THREAD;
 
 // Per kernel kind (one-seed pass, two-seed pass, update): how many 16-byte
 // vectors of its tile a thread processes at once (the group; each bf16 vector
