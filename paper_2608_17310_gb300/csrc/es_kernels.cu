@@ -170,15 +170,11 @@ __device__ __forceinline__ float add_acc(float theta, float acc, float inv_scale
   else return theta + acc;
 }
 
-// Philox words of block j for one seed. TileGen serves the blocks of a tile
-// that share the high counter word (per-tile constants, see philox_tile);
-// SchedGen does the same with the round keys read from a precomputed schedule
-// (kernel parameters or registers loaded from shared memory); AnyGen serves
-// any block. All give the same words.
-struct TileGen {
-  PhiloxTile t;
-  __device__ uint4 block(uint64_t j) const { return philox_block_tile(static_cast<uint32_t>(j), t); }
-};
+// Philox words of block j for one seed. SchedGen serves the blocks of a tile
+// that share the high counter word, with the round keys read from a
+// precomputed schedule (kernel parameters or registers loaded from shared
+// memory) and the tile's constants computed once; AnyGen serves any block. Both
+// give the same words.
 template <class Keys, bool kWideFirst = false>
 struct SchedGen {
   TileConst t;
@@ -192,12 +188,6 @@ struct AnyGen {
   PhiloxKey key;
   __device__ uint4 block(uint64_t j) const { return philox_block(j, key); }
 };
-
-template <bool kUniformHi>
-__device__ __forceinline__ auto make_gen(PhiloxKey key, uint32_t j_hi) {
-  if constexpr (kUniformHi) return TileGen{philox_tile(j_hi, key)};
-  else return AnyGen{key};
-}
 
 // Generator of one seed whose schedule is a kernel parameter.
 template <bool kUniformHi, bool kWideFirst = false>
@@ -737,19 +727,29 @@ noise_fill_vec_kernel(uint64_t j_first, uint64_t nblocks, const __grid_constant_
   }
 }
 
-// out[4t .. 4t+3] = Philox words of block block_base + t. Even and odd blocks
-// go through the two implementations of the rounds (general, and with the
-// per-tile constants of philox_tile); they give identical words, and this lets
-// a bit-exact check of this output cover both.
+// out[4t .. 4t+3] = Philox words of block block_base + t. Block j goes
+// through one of the four implementations of the rounds by j mod 4: the
+// general one (philox_block), the one with per-tile constants (philox_tile),
+// and the scheduled-key one the streaming kernels use, with high/low product
+// pairs in the first two rounds or 64-bit-result products throughout
+// (philox_block_rk). They give identical words, and this lets a bit-exact check
+// of this output cover all four.
 __global__ void __launch_bounds__(kBlockThreads)
-noise_bits_kernel(uint64_t block_base, uint64_t nblocks, PhiloxKey key, uint4* __restrict__ out) {
+noise_bits_kernel(uint64_t block_base, uint64_t nblocks, const __grid_constant__ PhiloxSched sched,
+                  uint4* __restrict__ out) {
+  const PhiloxKey key{sched.rk[0], sched.rk[1]};
   const uint64_t stride = static_cast<uint64_t>(gridDim.x) * blockDim.x;
   for (uint64_t t = static_cast<uint64_t>(blockIdx.x) * blockDim.x + threadIdx.x; t < nblocks;
        t += stride) {
     const uint64_t j = block_base + t;
-    out[t] = (j & 1) ? philox_block_tile(static_cast<uint32_t>(j),
-                                         philox_tile(static_cast<uint32_t>(j >> 32), key))
-                     : philox_block(j, key);
+    const uint32_t j_lo = static_cast<uint32_t>(j), j_hi = static_cast<uint32_t>(j >> 32);
+    const TileConst tc = tile_const(j_hi, sched.rk[0], sched.rk[3]);
+    switch (j & 3) {
+      case 0: out[t] = philox_block(j, key); break;
+      case 1: out[t] = philox_block_tile(j_lo, philox_tile(j_hi, key)); break;
+      case 2: out[t] = philox_block_rk<false>(j_lo, tc, sched.rk[1], sched.rk[2], sched.rk + 4); break;
+      default: out[t] = philox_block_rk<true>(j_lo, tc, sched.rk[1], sched.rk[2], sched.rk + 4);
+    }
   }
 }
 
@@ -859,7 +859,7 @@ cudaError_t launch_noise_bits(uint64_t seed, uint64_t block_base, uint64_t nbloc
                               uint32_t* out, cudaStream_t stream) {
   const uint64_t ctas = (nblocks + kBlockThreads - 1) / kBlockThreads;
   const int grid = persistent_grid(noise_bits_kernel, ctas);
-  noise_bits_kernel<<<grid, kBlockThreads, 0, stream>>>(block_base, nblocks, philox_key(seed),
+  noise_bits_kernel<<<grid, kBlockThreads, 0, stream>>>(block_base, nblocks, philox_sched(seed),
                                                         reinterpret_cast<uint4*>(out));
   return cudaGetLastError();
 }
