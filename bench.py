@@ -3,20 +3,23 @@
 synthetic parameter set shaped like the paper's workloads.
 
     python bench.py [--gpus N] [--steps K] [--warmup W] [--workload qwen27b]
-                    [--impl ours|reference] [--no-e2e] [--no-cpu-baseline]
+                    [--impl ours|reference] [--no-e2e] [--no-cpu-baseline] [--unfused]
     python bench.py --sweep [--populations 1,2,4,...] [--workload qwen4b]
     python bench.py --replay [--population N] [--generations K]
     python bench.py --antithetic
     python bench.py --generator [--gen-log2 31]
-    python bench.py --pipe-peaks
+    python bench.py --pipe-peaks [--probes name,name,...]
 
 Prints one JSON line (rank 0). `value` is measured with the inputs resident in
 HBM; `e2e` is the same metric with the parameters in pinned host memory and
 copied to the device and back inside every timed step. The reference arm
 (`--impl reference`) times the CPU oracle, on every host core, on a bounded
 sample of the same workload. The other modes time one part of the path each:
-es_update per population size, seed-log replay, antithetic generations and the
-noise generator alone. With --gpus N > 1 (under torchrun) every rank runs an independent
+es_update per population size, seed-log replay, antithetic generations, the
+noise generator alone and the register-only pipe probes. The roofline is the
+nominal integer-multiply rate (the FMA-heavy pipe's rate for Philox's
+products); each kernel is also reported against the kernels' own generator
+run in registers in the same process (`generator_frac`). With --gpus N > 1 (under torchrun) every rank runs an independent
 replica of the step (replicas only: the ES step has no exchange between GPUs
 besides N scalar rewards) and the slowest rank's time is reported.
 """
