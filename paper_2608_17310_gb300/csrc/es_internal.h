@@ -64,6 +64,22 @@ constexpr int kVecsPerThread = ES_VECS_PER_THREAD;
 #ifndef ES_NEAR_ONE_BRANCH
 #define ES_NEAR_ONE_BRANCH 1
 #endif
+// Software pipelining of the update's seed loop (1): seed i + 1's Philox
+// words are computed beside seed i's transform. The values are identical.
+// (The same schedule in the perturb/restore passes, over (vector, seed)
+// items, measured 2-4 % slower there and is not built.)
+#ifndef ES_UPDATE_PIPELINED
+#define ES_UPDATE_PIPELINED 1
+#endif
+// Round 0's Philox product (kPhiloxMulA times the low counter word) depends
+// on the counter alone: 0 computes it per block and seed; 1 once per block,
+// shared by every seed of a pass (the fused restore + perturb, the update's
+// seeds and its trailing perturb); 2 as 1, and in a tile inside its segment
+// stepped from the thread's first block by 64-bit additions of constants
+// instead of multiplied. The words are identical.
+#ifndef ES_ROUND0
+#define ES_ROUND0 1
+#endif
 // Seeds of the update's seed loop issued together (independent generator
 // work per element across seeds; the accumulation stays in ascending order).
 #ifndef ES_SEED_UNROLL
@@ -75,10 +91,13 @@ constexpr int kUpdateGroup = ES_UPDATE_GROUP;
 static_assert(kVecsPerThread % kAxpy1Group == 0 && kVecsPerThread % kAxpy2Group == 0 &&
                   kVecsPerThread % kUpdateGroup == 0,
               "groups divide the vectors of a tile");
-constexpr int axpy_min_blocks(bool two) {
-  return (two ? ES_AXPY2_MIN_BLOCKS : ES_AXPY1_MIN_BLOCKS) > 0
-             ? (two ? ES_AXPY2_MIN_BLOCKS : ES_AXPY1_MIN_BLOCKS)
-             : 1;
+constexpr int axpy_min_blocks(bool two, int vec_elems = 8) {
+  const int m = (two ? ES_AXPY2_MIN_BLOCKS : ES_AXPY1_MIN_BLOCKS) > 0
+                    ? (two ? ES_AXPY2_MIN_BLOCKS : ES_AXPY1_MIN_BLOCKS)
+                    : 1;
+  // FP8 vectors hold twice the elements (twice the Philox blocks per vector):
+  // at most 2 CTAs per SM, so their registers do not spill
+  return vec_elems > 8 && m > 2 ? 2 : m;
 }
 constexpr int update_min_blocks() { return ES_UPDATE_MIN_BLOCKS > 0 ? ES_UPDATE_MIN_BLOCKS : 1; }
 // Elements per 16-byte vector, per dtype.

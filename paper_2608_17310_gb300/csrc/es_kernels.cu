@@ -183,6 +183,10 @@ struct SchedGen {
   __device__ uint4 block(uint64_t j) const {
     return philox_block_rk<kWideFirst>(static_cast<uint32_t>(j), t, rk1, rk2, rk);
   }
+  // The same words from round 0's product (philox_round0 of the block's j_lo).
+  __device__ uint4 block_r0(Round0 p0) const {
+    return philox_block_r0<kWideFirst>(p0, t, rk1, rk2, rk);
+  }
 };
 struct AnyGen {
   PhiloxKey key;
@@ -209,39 +213,56 @@ enum class NoiseForm { kScalar, kPackedFma, kPacked };
 constexpr NoiseForm kAxpy1Form = static_cast<NoiseForm>(ES_AXPY1_FORM);
 constexpr NoiseForm kAxpy2Form = static_cast<NoiseForm>(ES_AXPY2_FORM);
 constexpr NoiseForm kUpdateForm = static_cast<NoiseForm>(ES_UPDATE_FORM);
+constexpr bool kUpdatePipelined = ES_UPDATE_PIPELINED != 0;
+constexpr int kRound0 = ES_ROUND0;
 // Near-one radius inputs: a rare branch (true) or a select per pair (false).
 constexpr bool kNearOneBranch = ES_NEAR_ONE_BRANCH != 0;
 
-// The pairs of Philox blocks j0 .. j0 + NB - 1 in polar form (r, cos, sin),
-// .x of each Polar2 the block's pair (x0, x1), .y its pair (x2, x3).
-template <NoiseForm kForm, int NB, class Gen>
-__device__ __forceinline__ void polar_blocks(const Gen& gen, uint64_t j0, Polar2 (&p)[NB]) {
-  constexpr bool kLogOnly = kNearOneBranch;
-  uint2 xa[NB];
-#pragma unroll
-  for (int b = 0; b < NB; ++b) {
-    const uint4 x = gen.block(j0 + b);
-    xa[b] = make_uint2(x.x, x.z);
-    if constexpr (kForm == NoiseForm::kPacked) {
-      p[b] = polar2_sq<kLogOnly>(x);
-    } else {
-      const Polar a = polar_sq<kLogOnly>(x.x, x.y), c = polar_sq<kLogOnly>(x.z, x.w);
-      p[b] = Polar2{make_float2(a.r, c.r), make_float2(a.c, c.c), make_float2(a.s, c.s)};
-    }
-  }
-  if constexpr (kLogOnly) fix_near_one<NB>(xa, p);
+// The radius of every pair, from its radius^2.
+template <int NB>
+__device__ __forceinline__ void polar_roots(Polar2 (&p)[NB]) {
 #pragma unroll
   for (int b = 0; b < NB; ++b) p[b].r = make_float2(sqrt_approx(p[b].r.x), sqrt_approx(p[b].r.y));
 }
 
-// f[k] += scale * eps[4 j0 + k] for the V elements of Philox blocks j0,
-// j0 + 1, ..., with scale folded into each pair's radius.
-template <NoiseForm kForm, int V, class Gen>
-__device__ __forceinline__ void add_scaled_noise(const Gen& gen, uint64_t j0, float scale,
-                                                 float (&f)[V]) {
+// The pairs of NB Philox blocks in polar form (r, cos, sin) from their words.
+template <NoiseForm kForm, int NB>
+__device__ __forceinline__ void polar_from_words(const uint4 (&x)[NB], Polar2 (&p)[NB]) {
+  constexpr bool kLogOnly = kNearOneBranch;
+  uint2 xa[NB];
+#pragma unroll
+  for (int b = 0; b < NB; ++b) {
+    xa[b] = make_uint2(x[b].x, x[b].z);
+    if constexpr (kForm == NoiseForm::kPacked) {
+      p[b] = polar2_sq<kLogOnly>(x[b]);
+    } else {
+      const Polar a = polar_sq<kLogOnly>(x[b].x, x[b].y), c = polar_sq<kLogOnly>(x[b].z, x[b].w);
+      p[b] = Polar2{make_float2(a.r, c.r), make_float2(a.c, c.c), make_float2(a.s, c.s)};
+    }
+  }
+  if constexpr (kLogOnly) fix_near_one<NB>(xa, p);
+  polar_roots<NB>(p);
+}
+
+// Words of Philox blocks j0 .. j0 + NB - 1.
+template <int NB, class Gen>
+__device__ __forceinline__ void philox_words(const Gen& gen, uint64_t j0, uint4 (&x)[NB]) {
+#pragma unroll
+  for (int b = 0; b < NB; ++b) x[b] = gen.block(j0 + b);
+}
+
+template <NoiseForm kForm, int NB, class Gen>
+__device__ __forceinline__ void polar_blocks(const Gen& gen, uint64_t j0, Polar2 (&p)[NB]) {
+  uint4 x[NB];
+  philox_words<NB>(gen, j0, x);
+  polar_from_words<kForm, NB>(x, p);
+}
+
+// f[k] += scale * eps[4 j0 + k] for the V elements of blocks whose polar
+// forms are pp[0 .. V / 4), with scale folded into each pair's radius.
+template <NoiseForm kForm, int V>
+__device__ __forceinline__ void apply_noise(const Polar2* pp, float scale, float (&f)[V]) {
   constexpr int NB = V / 4;
-  Polar2 pp[NB];
-  polar_blocks<kForm, NB>(gen, j0, pp);
 #pragma unroll
   for (int b = 0; b < NB; ++b) {
     const Polar2& p = pp[b];
@@ -263,6 +284,26 @@ __device__ __forceinline__ void add_scaled_noise(const Gen& gen, uint64_t j0, fl
       f[4 * b + 3] = hi.y;
     }
   }
+}
+
+// f[k] += scale * eps[4 j0 + k] for the V elements of Philox blocks j0,
+// j0 + 1, ..., with scale folded into each pair's radius.
+template <NoiseForm kForm, int V, class Gen>
+__device__ __forceinline__ void add_scaled_noise(const Gen& gen, uint64_t j0, float scale,
+                                                 float (&f)[V]) {
+  Polar2 pp[V / 4];
+  polar_blocks<kForm, V / 4>(gen, j0, pp);
+  apply_noise<kForm, V>(pp, scale, f);
+}
+
+// f[k] += scale * eps for the V elements of the Philox blocks whose words
+// are x.
+template <NoiseForm kForm, int V>
+__device__ __forceinline__ void add_scaled_noise_words(const uint4 (&x)[V / 4], float scale,
+                                                       float (&f)[V]) {
+  Polar2 pp[V / 4];
+  polar_from_words<kForm, V / 4>(x, pp);
+  apply_noise<kForm, V>(pp, scale, f);
 }
 
 // f <- round(round(f + s1 * eps) + s2 * eps) for one seed's noise, computed
@@ -383,14 +424,25 @@ __device__ __forceinline__ void axpy_tile(const TileRef<Io>& cur, uint4 (&v)[G],
   constexpr int kGroups = kVecsPerThread / G;
   constexpr int kStride = kBlockThreads * V;  // elements from one vector of a thread to the next
   const uint32_t j_hi = static_cast<uint32_t>((cur.index_base + cur.t0) >> 34);
-  // the one-seed pass is fastest with every Philox product 64-bit wide
-  const auto gen = sched_gen<kUniformHi, !kTwo>(a.s1, j_hi);
+  // the one-seed pass is fastest with every Philox product 64-bit wide (in
+  // FP8 storage, with twice the blocks per vector, that spills)
+  constexpr bool kWide1 = !kTwo && V <= 8;
+  const auto gen = sched_gen<kUniformHi, kWide1>(a.s1, j_hi);
   const auto gen2 = sched_gen<kUniformHi && kTwo && !kSame>(a.s2, j_hi);
   const float s1 = a.scale1 * cur.inv, s2 = a.scale2 * cur.inv;
   // the thread's first element of the tile, and its Philox block (index_base
   // is a multiple of 8 and t0 of the tile size, so the division is exact)
   typename Io::Scalar* const p = cur.base + cur.t0 + threadIdx.x * V;
   const uint64_t j_thread = ((cur.index_base + cur.t0) >> 2) + threadIdx.x * (V / 4);
+  // Round 0's product from the counter alone (kRound0): once per block for
+  // both seeds of the fused pass, and in a tile inside its segment stepped
+  // from the thread's first block (its blocks share the high counter word,
+  // so j_lo + d never wraps).
+  constexpr int NB = V / 4;
+  constexpr bool kR0 = kUniformHi && !kSame && (kRound0 >= 2 ? (kFull || kTwo) : kRound0 >= 1 && kTwo);
+  constexpr bool kR0Step = kR0 && kFull && kRound0 >= 2;
+  Round0 p0_thread{0u, 0u};
+  if constexpr (kR0Step) p0_thread = philox_round0<kWide1>(static_cast<uint32_t>(j_thread));
 #pragma unroll
   for (int grp = 0; grp < kGroups; ++grp) {
     uint4 nv[G];
@@ -417,6 +469,22 @@ __device__ __forceinline__ void axpy_tile(const TileRef<Io>& cur, uint4 (&v)[G],
       Io::unpack(v[q], f);
       if constexpr (kSame) {
         add_scaled_noise_twice<Io, V>(gen, j0, s1, s2, f);
+      } else if constexpr (kR0) {
+        Round0 p0[NB];
+#pragma unroll
+        for (int b = 0; b < NB; ++b)
+          p0[b] = kR0Step ? round0_step(p0_thread, static_cast<uint32_t>(u * (kStride / 4) + b))
+                          : philox_round0<kWide1>(static_cast<uint32_t>(j0 + b));
+        uint4 x[NB];
+#pragma unroll
+        for (int b = 0; b < NB; ++b) x[b] = gen.block_r0(p0[b]);
+        add_scaled_noise_words<kAxpyForm, V>(x, s1, f);
+        if constexpr (kTwo) {
+          Io::round_trip(f);
+#pragma unroll
+          for (int b = 0; b < NB; ++b) x[b] = gen2.block_r0(p0[b]);
+          add_scaled_noise_words<kAxpyForm, V>(x, s2, f);
+        }
       } else {
         add_scaled_noise<kAxpyForm, V>(gen, j0, s1, f);
         if constexpr (kTwo) {
@@ -444,7 +512,7 @@ __device__ __forceinline__ void axpy_tile(const TileRef<Io>& cur, uint4 (&v)[G],
 // For a scaled storage type (FP8) the noise is added in units of the
 // segment's scale: scale * inv_scale[segment].
 template <class Io, bool kTwo, bool kSame>
-__global__ void __launch_bounds__(kBlockThreads, axpy_min_blocks(kTwo))
+__global__ void __launch_bounds__(kBlockThreads, axpy_min_blocks(kTwo, Io::kVec))
 axpy_noise_kernel(const SegDesc* __restrict__ segs, const float* __restrict__ inv_scale,
                   uint64_t total_tiles, const __grid_constant__ AxpyArgs a) {
   constexpr int G = group_for<Io>(kTwo ? kAxpy2Group : kAxpy1Group);
@@ -555,15 +623,52 @@ __device__ __forceinline__ void accumulate_seeds(const TileRef<Io>& r, int u0, c
                                                  int count, float (&acc)[G][Io::kVec]) {
   constexpr int V = Io::kVec;
   constexpr int kUnroll = ES_SEED_UNROLL;
-#pragma unroll kUnroll
-  for (int i = 0; i < count; ++i) {
-    const auto gen = row_gen<kUniformHi>(rows[i]);
-    const float c = row_coeff(rows[i]);
+  if constexpr (kUpdatePipelined && G == 1 && V <= 8) {
+    // Software-pipelined over the seeds: seed i + 1's Philox words are
+    // computed in the same basic block as seed i's transform, so the
+    // integer-multiply phase of one seed overlaps the MUFU/FP32 phase of the
+    // other.
+    constexpr int NB = V / 4;
+    const uint64_t e = vec_elem(r, u0);
+    if (e >= r.numel || count < 1) return;
+    const uint64_t j0 = (r.index_base + e) >> 2;
+    // round 0's products, shared by every seed (kRound0)
+    constexpr bool kR0 = kUniformHi && kRound0 >= 1;
+    Round0 p0[NB];
 #pragma unroll
-    for (int q = 0; q < G; ++q) {
-      const uint64_t e = vec_elem(r, u0 + q);
-      if (e >= r.numel) continue;
-      add_scaled_noise<kUpdateForm, V>(gen, (r.index_base + e) >> 2, c, acc[q]);
+    for (int b = 0; b < NB; ++b)
+      p0[b] = kR0 ? philox_round0<false>(static_cast<uint32_t>(j0 + b)) : Round0{0u, 0u};
+    auto words = [&](const SchedRow& row, uint4 (&w)[NB]) {
+      const auto gen = row_gen<kUniformHi>(row);
+#pragma unroll
+      for (int b = 0; b < NB; ++b) {
+        if constexpr (kR0) w[b] = gen.block_r0(p0[b]);
+        else w[b] = gen.block(j0 + b);
+      }
+    };
+    uint4 x[NB];
+    words(rows[0], x);
+    auto transform = [&](float c) { add_scaled_noise_words<kUpdateForm, V>(x, c, acc[0]); };
+#pragma unroll 1
+    for (int i = 0; i + 1 < count; ++i) {
+      uint4 xn[NB];
+      words(rows[i + 1], xn);
+      transform(row_coeff(rows[i]));
+#pragma unroll
+      for (int b = 0; b < NB; ++b) x[b] = xn[b];
+    }
+    transform(row_coeff(rows[count - 1]));
+  } else {
+#pragma unroll kUnroll
+    for (int i = 0; i < count; ++i) {
+      const auto gen = row_gen<kUniformHi>(rows[i]);
+      const float c = row_coeff(rows[i]);
+#pragma unroll
+      for (int q = 0; q < G; ++q) {
+        const uint64_t e = vec_elem(r, u0 + q);
+        if (e >= r.numel) continue;
+        add_scaled_noise<kUpdateForm, V>(gen, (r.index_base + e) >> 2, c, acc[q]);
+      }
     }
   }
 }
@@ -731,9 +836,11 @@ noise_fill_vec_kernel(uint64_t j_first, uint64_t nblocks, const __grid_constant_
 // through one of the four implementations of the rounds by j mod 4: the
 // general one (philox_block), the one with per-tile constants (philox_tile),
 // and the scheduled-key one the streaming kernels use, with high/low product
-// pairs in the first two rounds or 64-bit-result products throughout
-// (philox_block_rk). They give identical words, and this lets a bit-exact check
-// of this output cover all four.
+// pairs in the first two rounds (philox_block_rk), or with 64-bit-result
+// products throughout and round 0's product stepped from that of a lower
+// counter word by 64-bit additions (round0_step, philox_block_r0). They give
+// identical words, and this lets a bit-exact check of this output cover all
+// four.
 __global__ void __launch_bounds__(kBlockThreads)
 noise_bits_kernel(uint64_t block_base, uint64_t nblocks, const __grid_constant__ PhiloxSched sched,
                   uint4* __restrict__ out) {
@@ -748,7 +855,11 @@ noise_bits_kernel(uint64_t block_base, uint64_t nblocks, const __grid_constant__
       case 0: out[t] = philox_block(j, key); break;
       case 1: out[t] = philox_block_tile(j_lo, philox_tile(j_hi, key)); break;
       case 2: out[t] = philox_block_rk<false>(j_lo, tc, sched.rk[1], sched.rk[2], sched.rk + 4); break;
-      default: out[t] = philox_block_rk<true>(j_lo, tc, sched.rk[1], sched.rk[2], sched.rk + 4);
+      default: {
+        // from j_lo rounded down to a multiple of 2^11, d = j_lo mod 2^11 (no wrap)
+        const Round0 p0 = round0_step(philox_round0<true>(j_lo & ~0x7FFu), j_lo & 0x7FFu);
+        out[t] = philox_block_r0<true>(p0, tc, sched.rk[1], sched.rk[2], sched.rk + 4);
+      }
     }
   }
 }

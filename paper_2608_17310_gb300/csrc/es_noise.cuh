@@ -156,18 +156,48 @@ __device__ __forceinline__ TileConst tile_const(uint32_t j_hi, uint32_t k0, uint
 // kernel). Bit-identical to philox_block.
 template <bool kWideFirst, class Keys>
 __device__ __forceinline__ uint4 philox_block_rk(uint32_t j_lo, TileConst t, uint32_t rk1,
+                                                 uint32_t rk2, const Keys& rk);
+
+// Round 0's product kPhiloxMulA * j_lo as (high, low) words. It depends on
+// the counter alone, not on the key: every seed's block j shares it.
+struct Round0 {
+  uint32_t hi, lo;
+};
+
+template <bool kWide>
+__device__ __forceinline__ Round0 philox_round0(uint32_t j_lo) {
+  Round0 p;
+  if constexpr (kWide) {
+    mul_wide(kPhiloxMulA, j_lo, p.hi, p.lo);
+  } else {
+    p.hi = mul_hi(kPhiloxMulA, j_lo);
+    p.lo = mul_lo(kPhiloxMulA, j_lo);
+  }
+  return p;
+}
+
+// The product of round 0 for counter word j_lo + d, from the one for j_lo:
+// the 64-bit product grows by kPhiloxMulA * d. Exact while j_lo + d stays
+// below 2^32 (the caller's blocks share their high counter word).
+__device__ __forceinline__ Round0 round0_step(Round0 p, uint32_t d) {
+  const uint64_t q = ((static_cast<uint64_t>(p.hi) << 32) | p.lo) +
+                     static_cast<uint64_t>(kPhiloxMulA) * d;
+  return Round0{static_cast<uint32_t>(q >> 32), static_cast<uint32_t>(q)};
+}
+
+// philox_block_rk from round 0's product (philox_round0 of the block's j_lo).
+template <bool kWideFirst, class Keys>
+__device__ __forceinline__ uint4 philox_block_r0(Round0 p0, TileConst t, uint32_t rk1,
                                                  uint32_t rk2, const Keys& rk) {
-  uint32_t a2, a3, c0, c1;
+  const uint32_t a2 = p0.hi ^ rk1;  // round 0: word 2 (its word 3 is p0.lo)
+  const uint32_t a3 = p0.lo;
+  uint32_t c0, c1;
   if constexpr (kWideFirst) {
-    uint32_t h0, h1;
-    mul_wide(kPhiloxMulA, j_lo, h0, a3);  // round 0: words 2 and 3
-    a2 = h0 ^ rk1;
-    mul_wide(kPhiloxMulB, a2, h1, c1);    // round 1 (its word 1 was 0)
+    uint32_t h1;
+    mul_wide(kPhiloxMulB, a2, h1, c1);  // round 1 (its word 1 was 0)
     c0 = h1 ^ rk2;
   } else {
-    a2 = mul_hi(kPhiloxMulA, j_lo) ^ rk1;  // round 0, word 2
-    a3 = mul_lo(kPhiloxMulA, j_lo);        // round 0, word 3
-    c0 = mul_hi(kPhiloxMulB, a2) ^ rk2;    // round 1 (its word 1 was 0)
+    c0 = mul_hi(kPhiloxMulB, a2) ^ rk2;  // round 1 (its word 1 was 0)
     c1 = mul_lo(kPhiloxMulB, a2);
   }
   uint32_t c2 = t.x2 ^ a3;
@@ -185,6 +215,12 @@ __device__ __forceinline__ uint4 philox_block_rk(uint32_t j_lo, TileConst t, uin
     c2 = n2;
   }
   return make_uint4(c0, c1, c2, c3);
+}
+
+template <bool kWideFirst, class Keys>
+__device__ __forceinline__ uint4 philox_block_rk(uint32_t j_lo, TileConst t, uint32_t rk1,
+                                                 uint32_t rk2, const Keys& rk) {
+  return philox_block_r0<kWideFirst>(philox_round0<kWideFirst>(j_lo), t, rk1, rk2, rk);
 }
 
 // The float 1 + m 2^-23 for m = x >> 9 (the top 23 bits of x).
