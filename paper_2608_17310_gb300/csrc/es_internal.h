@@ -78,7 +78,7 @@ constexpr int kVecsPerThread = ES_VECS_PER_THREAD;
 // stepped from the thread's first block by 64-bit additions of constants
 // instead of multiplied. The words are identical.
 #ifndef ES_ROUND0
-#define ES_ROUND0 1
+#define ES_ROUND0 2
 #endif
 // Seeds of the update's seed loop issued together (independent generator
 // work per element across seeds; the accumulation stays in ascending order).
