@@ -64,12 +64,14 @@ constexpr int kVecsPerThread = ES_VECS_PER_THREAD;
 #ifndef ES_NEAR_ONE_BRANCH
 #define ES_NEAR_ONE_BRANCH 1
 #endif
-// Software pipelining of the update's seed loop (1): seed i + 1's Philox
-// words are computed beside seed i's transform. The values are identical.
+// Software pipelining of the update's seed loop: seed i + 1's Philox words
+// are computed beside seed i's transform (1: one seed per iteration, the
+// words copied to the next iteration's buffer; 2: two seeds per iteration
+// on alternating buffers). The values are identical.
 // (The same schedule in the perturb/restore passes, over (vector, seed)
 // items, measured 2-4 % slower there and is not built.)
 #ifndef ES_UPDATE_PIPELINED
-#define ES_UPDATE_PIPELINED 1
+#define ES_UPDATE_PIPELINED 2
 #endif
 // Round 0's Philox product (kPhiloxMulA times the low counter word) depends
 // on the counter alone: 0 computes it per block and seed; 1 once per block,

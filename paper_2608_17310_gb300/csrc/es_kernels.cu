@@ -32,11 +32,13 @@ struct Bf16Io {
     __nv_bfloat162 h = __floats2bfloat162_rn(lo, hi);  // one cvt.rn.bf16x2.f32
     return *reinterpret_cast<uint32_t*>(&h);
   }
+  __device__ static float lo(uint32_t w) { return __uint_as_float(w << 16); }
+  __device__ static float hi(uint32_t w) { return __uint_as_float(w & 0xFFFF0000u); }
   __device__ static void unpack(const uint4& v, float (&f)[8]) {
-    f[0] = __uint_as_float(v.x << 16); f[1] = __uint_as_float(v.x & 0xFFFF0000u);
-    f[2] = __uint_as_float(v.y << 16); f[3] = __uint_as_float(v.y & 0xFFFF0000u);
-    f[4] = __uint_as_float(v.z << 16); f[5] = __uint_as_float(v.z & 0xFFFF0000u);
-    f[6] = __uint_as_float(v.w << 16); f[7] = __uint_as_float(v.w & 0xFFFF0000u);
+    f[0] = lo(v.x); f[1] = hi(v.x);
+    f[2] = lo(v.y); f[3] = hi(v.y);
+    f[4] = lo(v.z); f[5] = hi(v.z);
+    f[6] = lo(v.w); f[7] = hi(v.w);
   }
   __device__ static uint4 pack(const float (&f)[8]) {
     return make_uint4(pack2(f[0], f[1]), pack2(f[2], f[3]), pack2(f[4], f[5]), pack2(f[6], f[7]));
@@ -47,8 +49,8 @@ struct Bf16Io {
 #pragma unroll
     for (int k = 0; k < M; k += 2) {
       const uint32_t w = pack2(f[k], f[k + 1]);
-      f[k] = __uint_as_float(w << 16);
-      f[k + 1] = __uint_as_float(w & 0xFFFF0000u);
+      f[k] = lo(w);
+      f[k + 1] = hi(w);
     }
   }
   // The first `rem` (< 8) elements at base[e], the rest zero, as one vector.
@@ -214,6 +216,7 @@ constexpr NoiseForm kAxpy1Form = static_cast<NoiseForm>(ES_AXPY1_FORM);
 constexpr NoiseForm kAxpy2Form = static_cast<NoiseForm>(ES_AXPY2_FORM);
 constexpr NoiseForm kUpdateForm = static_cast<NoiseForm>(ES_UPDATE_FORM);
 constexpr bool kUpdatePipelined = ES_UPDATE_PIPELINED != 0;
+constexpr bool kUpdatePingPong = ES_UPDATE_PIPELINED >= 2;
 constexpr int kRound0 = ES_ROUND0;
 // Near-one radius inputs: a rare branch (true) or a select per pair (false).
 constexpr bool kNearOneBranch = ES_NEAR_ONE_BRANCH != 0;
@@ -646,18 +649,40 @@ __device__ __forceinline__ void accumulate_seeds(const TileRef<Io>& r, int u0, c
         else w[b] = gen.block(j0 + b);
       }
     };
+    auto transform = [&](const uint4 (&w)[NB], const SchedRow& row) {
+      add_scaled_noise_words<kUpdateForm, V>(w, row_coeff(row), acc[0]);
+    };
     uint4 x[NB];
     words(rows[0], x);
-    auto transform = [&](float c) { add_scaled_noise_words<kUpdateForm, V>(x, c, acc[0]); };
+    if constexpr (kUpdatePingPong) {
+      // two seeds per iteration, the word buffers alternating, so no copies
+      uint4 y[NB];
+      int i = 0;
 #pragma unroll 1
-    for (int i = 0; i + 1 < count; ++i) {
-      uint4 xn[NB];
-      words(rows[i + 1], xn);
-      transform(row_coeff(rows[i]));
+      for (; i + 2 < count; i += 2) {
+        words(rows[i + 1], y);
+        transform(x, rows[i]);
+        words(rows[i + 2], x);
+        transform(y, rows[i + 1]);
+      }
+      if (i + 1 < count) {
+        words(rows[i + 1], y);
+        transform(x, rows[i]);
+        transform(y, rows[i + 1]);
+      } else {
+        transform(x, rows[i]);
+      }
+    } else {
+#pragma unroll 1
+      for (int i = 0; i + 1 < count; ++i) {
+        uint4 xn[NB];
+        words(rows[i + 1], xn);
+        transform(x, rows[i]);
 #pragma unroll
-      for (int b = 0; b < NB; ++b) x[b] = xn[b];
+        for (int b = 0; b < NB; ++b) x[b] = xn[b];
+      }
+      transform(x, rows[count - 1]);
     }
-    transform(row_coeff(rows[count - 1]));
   } else {
 #pragma unroll kUnroll
     for (int i = 0; i < count; ++i) {
