@@ -77,8 +77,8 @@ __device__ __forceinline__ uint4 philox_block(uint64_t j, PhiloxKey key) {
 // Bit-identical to philox_block.
 struct PhiloxTile {
   PhiloxKey key;
-  uint32_t w0;     // word 0 after round 1: j_hi ^ k0
-  uint32_t x2;     // high word of kPhiloxMulA * w0, xored with round 2's k1
+  uint32_t w0;     // word 0 after round 0: j_hi ^ k0
+  uint32_t x2;     // high word of kPhiloxMulA * w0, xored with round 1's k1
   uint32_t lo2;    // low word of kPhiloxMulA * w0
 };
 
@@ -89,10 +89,10 @@ __device__ __forceinline__ PhiloxTile philox_tile(uint32_t j_hi, PhiloxKey key) 
 }
 
 __device__ __forceinline__ uint4 philox_block_tile(uint32_t j_lo, const PhiloxTile& t) {
-  // round 1 (keys k0, k1): products kPhiloxMulA * j_lo and kPhiloxMulB * 0
+  // round 0 (keys k0, k1): products kPhiloxMulA * j_lo and kPhiloxMulB * 0
   const uint32_t a2 = mul_hi(kPhiloxMulA, j_lo) ^ t.key.k1;   // word 2
   const uint32_t a3 = mul_lo(kPhiloxMulA, j_lo);              // word 3
-  // round 2 (keys k0 + W_A, k1 + W_B): word 0 is t.w0, its product is per tile
+  // round 1 (keys k0 + W_A, k1 + W_B): word 0 is t.w0, its product is per tile
   uint32_t c0 = mul_hi(kPhiloxMulB, a2) ^ (t.key.k0 + kPhiloxWeylA);  // word 1 was 0
   uint32_t c1 = mul_lo(kPhiloxMulB, a2);
   uint32_t c2 = t.x2 ^ a3;
