@@ -1091,24 +1091,33 @@ def e2e_fits(torch, nbytes: int, dist) -> bool:
 
 def copy_groups(sizes, groups=8):
     """Ends (exclusive tensor indices) of the contiguous copy groups of the e2e
-    leg. The last group holds the trailing tensors up to 1/32 of the elements
-    (at least one tensor): its copy back after the last update and its first
-    pass after the last copy in are the parts no other work hides. The rest is
-    split into groups - 1 groups of about equal size."""
+    leg. A group's copy back (and its copy in for the next step) starts when
+    its last pass is done, so whatever copying is left when the last pass of
+    the step ends is exposed. The groups therefore shrink towards the end: the
+    last holds the trailing tensors up to 1/32 of the elements (at least one
+    tensor), and each group before it up to twice as much as the one after it,
+    while that stays below 1/groups of the elements; the tensors before them
+    are split into groups of about 1/groups of the elements each. A tail group's
+    round trip then overlaps the last passes of the groups after it."""
     total = sum(sizes)
-    tail, acc = len(sizes), 0
-    while tail > 1 and (acc == 0 or acc + sizes[tail - 1] <= total / 32):
-        tail -= 1
-        acc += sizes[tail]
+    share = total / groups
+    tail_ends, end, cap = [], len(sizes), total / 32
+    while end > 1 and cap < share:
+        start, acc = end, 0
+        while start > 1 and (acc == 0 or acc + sizes[start - 1] <= cap):
+            start -= 1
+            acc += sizes[start]
+        tail_ends.append(end)
+        end = start
+        cap = max(2 * cap, 2 * acc)
+    head = sum(sizes[:end])
+    nhead = max(1, round(head / share))
     ends, acc = [], 0
-    head = sum(sizes[:tail])
-    for k in range(tail):
+    for k in range(end):
         acc += sizes[k]
-        if acc >= head * (len(ends) + 1) / max(groups - 1, 1) or k == tail - 1:
+        if acc >= head * (len(ends) + 1) / nhead or k == end - 1:
             ends.append(k + 1)
-    if tail < len(sizes):
-        ends.append(len(sizes))
-    return ends
+    return ends + tail_ends[::-1]
 
 
 class E2ELoop:
@@ -1124,10 +1133,10 @@ class E2ELoop:
     call is elementwise (tested)."""
 
     def __init__(self, torch, es, plan, flat, params, wl, n, esize, sigma_at, s_handle, fused,
-                 groups=8, nstreams=4):
+                 groups=8, nstreams=4, lead=2):
         self.torch, self.es, self.plan, self.flat = torch, es, plan, flat
         self.wl, self.n, self.sigma_at, self.s_handle, self.fused = wl, n, sigma_at, s_handle, fused
-        self.nstreams = nstreams
+        self.nstreams, self.lead = nstreams, lead
         self.pending = None  # per group: the event of its copy in issued by the previous step
         # The first use of a fresh page-locked buffer sometimes splits some of
         # its huge pages, and copies through it then run 5-9x slower (the
@@ -1175,6 +1184,23 @@ class E2ELoop:
             done.record(cs)
         return done
 
+    def passes(self, seeds, sigma):
+        """The generation's passes before its last one, in order, as
+        (call, arguments after the plan) pairs."""
+        es, n, sh = self.es, self.n, self.s_handle
+        out = []
+        if self.fused:
+            # the previous step's last pass perturbed with seeds[0]
+            for i in range(1, n):
+                out.append((es.es_restore_perturb,
+                            (int(seeds[i - 1]), sigma, int(seeds[i]), sigma, sh)))
+            out.append((es.es_restore, (int(seeds[n - 1]), sigma, sh)))
+        else:
+            for i in range(n):
+                out.append((es.es_perturb, (int(seeds[i]), sigma, sh)))
+                out.append((es.es_restore, (int(seeds[i]), sigma, sh)))
+        return out
+
     def step(self, t, record=None, copy_next=False):
         torch, es, plan = self.torch, self.es, self.plan
         wl, n, sh, stream = self.wl, self.n, self.s_handle, self.stream
@@ -1183,7 +1209,7 @@ class E2ELoop:
         ev = [torch.cuda.Event(enable_timing=True) for _ in range(4)]
         ev[0].record(stream)
         # in: unless the previous step already issued them, every copy waits
-        # only for the previous step; each group's first pass waits only for
+        # only for the previous step; each group's first passes wait only for
         # its own copy
         if self.pending is None:
             for cs in self.copy_streams:
@@ -1191,26 +1217,18 @@ class E2ELoop:
             landed = [self._copy_in(g) for g in range(len(self.spans))]
         else:
             landed, self.pending = self.pending, None
+        # the first `lead` passes group by group, so that the groups copied
+        # last (the smallest) get the earlier groups' passes to land in; the
+        # rest on the whole plan
+        todo = self.passes(seeds, sigma)
+        lead = min(self.lead, len(todo))
         for (a, b, gplan), done in zip(self.spans, landed):
             stream.wait_event(done)
-            if not self.fused:
-                es.es_perturb(gplan, int(seeds[0]), sigma, sh)
-            elif n > 1:
-                es.es_restore_perturb(gplan, int(seeds[0]), sigma, int(seeds[1]), sigma, sh)
-            else:
-                es.es_restore(gplan, int(seeds[0]), sigma, sh)
+            for call, rest in todo[:lead]:
+                call(gplan, *rest)
         ev[1].record(stream)
-        # middle of the generation on the whole plan
-        if self.fused:
-            for i in range(2, n):
-                es.es_restore_perturb(plan, int(seeds[i - 1]), sigma, int(seeds[i]), sigma, sh)
-            if n > 1:
-                es.es_restore(plan, int(seeds[n - 1]), sigma, sh)
-        else:
-            es.es_restore(plan, int(seeds[0]), sigma, sh)
-            for i in range(1, n):
-                es.es_perturb(plan, int(seeds[i]), sigma, sh)
-                es.es_restore(plan, int(seeds[i]), sigma, sh)
+        for call, rest in todo[lead:]:
+            call(plan, *rest)
         coeffs = es.es_update_coeffs(es.es_normalize_rewards(rewards, 1e-8), wl.alpha, sigma,
                                      es.ES_SCALE_PAPER)
         first_next = int(generation_inputs(wl, t + 1, n)[0][0])
@@ -1273,12 +1291,14 @@ def run_e2e(args, torch, es, plan, flat, params, wl, n, esize, sigma_at, s_handl
     e1.record(stream)
     torch.cuda.synchronize()
     ms = max_over_ranks(e0.elapsed_time(e1), dist)
-    phases = {"copy_in_and_first_pass": 0.0, "middle_passes": 0.0, "last_pass_and_copy_out": 0.0}
+    phases = {"copy_in_and_first_passes": 0.0, "middle_passes": 0.0,
+              "last_pass_and_copy_out": 0.0}
     for ev in evs:
-        for name, a, b in (("copy_in_and_first_pass", 0, 1), ("middle_passes", 1, 2),
+        for name, a, b in (("copy_in_and_first_passes", 0, 1), ("middle_passes", 1, 2),
                            ("last_pass_and_copy_out", 2, 3)):
             phases[name] += ev[a].elapsed_time(ev[b]) / len(evs)
     kind, ngroups, bytes_per_copy = loop.pinned.kind, len(loop.spans), loop.bytes_per_copy
+    lead = loop.lead
     huge = loop.pinned.hugepage_fraction()
     hp_fault = loop.pinned.hugepages_at_registration
     attempts = loop.attempts
@@ -1292,9 +1312,10 @@ def run_e2e(args, torch, es, plan, flat, params, wl, n, esize, sigma_at, s_handl
             "host_buffer_attempts": attempts,
             "layout": f"one page-locked host buffer ({kind}) and one device buffer "
                       f"holding every tensor; {ngroups} groups with a plan each, copies over "
-                      f"{nstreams} streams; a group's copy back and its copy in for the next "
-                      f"step run while the other groups' last passes compute, and its first "
-                      f"pass waits only for its own copy"}
+                      f"{nstreams} streams, the groups shrinking towards the end; a group's "
+                      f"copy back and its copy in for the next step run while the other "
+                      f"groups' last passes compute, and its first {lead} passes (group by "
+                      f"group) wait only for its own copy"}
 
 
 # --- CPU oracle (cpu_baseline leg and the reference arm) ---------------------------------

@@ -70,14 +70,25 @@ def test_hugepage_fraction_of_an_anonymous_mapping_is_a_fraction():
     assert buf.hugepage_fraction() is None
 
 
-def test_copy_groups_cover_every_tensor_with_a_small_last_group():
+def test_copy_groups_cover_every_tensor_with_a_shrinking_tail():
     from paper_2608_17310_gb300 import inputs as I
     for name in ("qwen27b", "qwen4b", "qwen4b_4layer", "toy"):
         sizes = [s.numel for s in I.shapes_for(name)]
+        total = sum(sizes)
         ends = bench.copy_groups(sizes, 8)
-        assert ends[-1] == len(sizes) and len(ends) <= 8
-        assert all(b > a for a, b in zip([0] + ends[:-1], ends))   # non-empty, in order
-        last = sizes[(ends[-2] if len(ends) > 1 else 0):]
-        assert len(last) == 1 or sum(last) <= sum(sizes) / 32
+        starts = [0] + ends[:-1]
+        assert ends[-1] == len(sizes) and len(ends) <= 12
+        assert all(b > a for a, b in zip(starts, ends))   # non-empty, in order
+        group = [sum(sizes[a:b]) for a, b in zip(starts, ends)]
+        # the last group: at most 1/32 of the elements, or a single tensor
+        assert ends[-1] - starts[-1] == 1 or group[-1] <= total / 32
+    # on the 27B-shaped set the groups shrink towards the end: each of the
+    # last three at most half the one before it (within one tensor)
+    sizes = [s.numel for s in I.shapes_for("qwen27b")]
+    ends = bench.copy_groups(sizes, 8)
+    starts = [0] + ends[:-1]
+    group = [sum(sizes[a:b]) for a, b in zip(starts, ends)]
+    big = max(sizes)
+    assert group[-1] <= group[-2] and group[-2] <= group[-3] / 2 + big
     assert bench.copy_groups([5], 8) == [1]
     assert bench.copy_groups([1] * 64, 8)[-1] == 64

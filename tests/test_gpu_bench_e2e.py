@@ -1,7 +1,7 @@
 """The e2e leg of bench.py computes exactly the generation it times: its
-grouped schedule (copy in, first pass per group plan, middle passes on the
-whole plan, last pass per group plan, copy out, and with pipelining the next
-step's copy in right after each group's copy out) leaves, after three
+grouped schedule (copy in, the first passes group by group, middle passes on
+the whole plan, last pass per group plan, copy out, and with pipelining the
+next step's copy in right after each group's copy out) leaves, after three
 generations, the host buffer and the device buffer bit-identical to the
 whole-plan loop that the device-timed leg runs."""
 import numpy as np
