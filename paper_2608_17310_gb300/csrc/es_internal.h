@@ -27,9 +27,12 @@ constexpr int kVecsPerThread = ES_VECS_PER_THREAD;
 // (0 scalar FP32, 1 scalar transform with packed FMAs, 2 packed; the values
 // are bit-identical). Measured on sm_103a over the 4B-shaped set: one vector
 // at a time is fastest for every kernel, at 2 CTAs per SM (128 registers) for
-// the two-seed pass and 3 for the others; more CTAs per SM, larger groups or a
-// second seed in flight gain nothing, since the generator is bound by the
-// FMA-heavy pipe (its integer products and packed FP32), not by latency.
+// the two-seed pass and 3 for the others; more CTAs per SM or larger groups
+// gain nothing, since the generator is bound by the FMA-heavy pipe (its
+// integer products and packed FP32), not by latency. What does gain is
+// interleaving the phases of independent work in one basic block: the
+// update's seed loop computes the next seed's Philox words beside the current
+// seed's transform (ES_UPDATE_PIPELINED).
 #ifndef ES_AXPY1_GROUP
 #define ES_AXPY1_GROUP 1
 #endif
