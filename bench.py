@@ -477,6 +477,7 @@ def run_ours(args, rank, world, dist):
     imul_peak, gauss_peak, gen_peak, sms, sm_max_mhz, hbm_gbs, peak_src, ceilings = \
         alu_peaks(torch, dev_index)
     bytes_per_launch = 2 * esize * P
+    gen_pipe = ceilings["generator_pipelined"]["gauss_per_s"]
     kernels = {}
     for name in timers.names():
         mean = timers.mean_ms(name)
@@ -488,6 +489,7 @@ def run_ours(args, rank, world, dist):
                          "mean_ms": mean, "share": timers.total_ms(name) / ms,
                          "gbs": gbs, "gauss_per_s": gps, "hbm_frac": hbm_frac,
                          "alu_frac": alu_frac, "generator_frac": gps / gen_peak,
+                         "generator_pipelined_frac": gps / gen_pipe,
                          "bound": "alu" if alu_frac > hbm_frac else "hbm"}
     dom = max(kernels, key=lambda k: kernels[k]["share"])
     d = kernels[dom]
@@ -508,7 +510,11 @@ def run_ours(args, rank, world, dist):
         "source": "measured in this run: the kernels' own generator (Philox, Box-Muller) in a "
                   "register-only loop with no memory traffic, 4 CTAs per SM, scaled to the "
                   "maximum SM clock: what this instruction stream reaches on its own "
-                  "(bench.py --pipe-peaks has every probe)"}
+                  "(bench.py --pipe-peaks has every probe)",
+        "pipelined": {"gauss_per_s": gen_pipe, "frac": d["gauss_per_s"] / gen_pipe,
+                      "source": "the same generator with two seeds' blocks alternating, the "
+                                "next seed's Philox words beside the current seed's transform, "
+                                "as in the update's seed loop"}}
     roof["measured_ceilings"] = ceilings
     roof["pipe_occupancy"] = pipe_occupancy(dom)
     roof.update({"kernel": d["kernel"], "hbm_frac": d["hbm_frac"], "alu_frac": d["alu_frac"],
@@ -597,7 +603,10 @@ def measured_ceilings(res, sms, sm_max_mhz):
       generator      the streaming kernels' generator (Philox with scheduled
                      round keys, the packed transform, the near-one series on a
                      rare branch) in registers, no memory traffic: the rate this
-                     instruction stream reaches on its own."""
+                     instruction stream reaches on its own;
+      generator_pipelined  the same generator with two seeds' blocks
+                     alternating, the next seed's Philox words computed beside
+                     the current seed's transform (the update's seed loop)."""
     hz = sms * sm_max_mhz * 1e6
     out = {}
     for name, per_g in (("imad_wide", WIDE_PER_GAUSS), ("lop3", LOP3_PER_GAUSS),
@@ -620,6 +629,9 @@ def measured_ceilings(res, sms, sm_max_mhz):
     if "generator" in res:
         r = res["generator"]["ops_per_clk_sm"]
         out["generator"] = {"gauss_per_clk_sm": r, "gauss_per_s": r * hz}
+    if "generator_pipelined" in res:
+        r = res["generator_pipelined"]["ops_per_clk_sm"]
+        out["generator_pipelined"] = {"gauss_per_clk_sm": r, "gauss_per_s": r * hz}
     if all(k in res for k in ("split_imad_wide_only", "split_mufu_only", "split_both")):
         ti = res["split_imad_wide_only"]["cycles"]
         tm = res["split_mufu_only"]["cycles"]
@@ -630,7 +642,7 @@ def measured_ceilings(res, sms, sm_max_mhz):
 
 
 CEILING_PROBES = ("imad_wide", "lop3", "mufu", "mix_imad_wide_mufu_9_4", "mix_imad_hi_lo_1_1",
-                  "mix_imad_hi_lo_mufu_9_4", "generator")
+                  "mix_imad_hi_lo_mufu_9_4", "generator", "generator_pipelined")
 
 
 def alu_peaks(torch, dev_index, probes=True):
@@ -685,7 +697,7 @@ def run_pipe_peaks(args, rank, world, dist):
         for name in names:
             res[name] = run_probe(L, name, 4, 25.0)
         for name in ("imad_wide", "mufu", "mix_imad_wide_mufu_9_4", "mix_imad_hi_lo_1_1",
-                     "mix_imad_hi_lo_mufu_9_4", "philox", "generator"):
+                     "mix_imad_hi_lo_mufu_9_4", "philox", "generator", "generator_pipelined"):
             if args.probes:
                 break
             for ctas in (1, 2, 8):
@@ -719,8 +731,9 @@ def run_sweep(args, rank, world, dist):
     P = plan.numel
     stream = torch.cuda.current_stream()
     s_handle = stream.cuda_stream
-    imul_peak, gauss_peak, gen_peak, sms, sm_max_mhz, hbm_gbs, peak_src, _ = \
+    imul_peak, gauss_peak, gen_peak, sms, sm_max_mhz, hbm_gbs, peak_src, ceilings = \
         alu_peaks(torch, dev_index)
+    gen_pipe = ceilings["generator_pipelined"]["gauss_per_s"]
     bytes_per_launch = 2 * esize * P
     pops = [int(x) for x in args.populations.split(",") if x.strip()]
     points = []
@@ -755,7 +768,7 @@ def run_sweep(args, rank, world, dist):
             points.append({
                 "population": n, "mean_ms": ms, "gbs": gbs, "gauss_per_s": gps,
                 "hbm_frac": gbs / hbm_gbs, "alu_frac": gps / gauss_peak,
-                "generator_frac": gps / gen_peak,
+                "generator_frac": gps / gen_peak, "generator_pipelined_frac": gps / gen_pipe,
                 "bound": "alu" if t_imul > t_hbm else "hbm",
                 "roofline_frac": max(t_hbm, t_imul) / ms,
                 "t_hbm_ms": t_hbm, "t_imul_ms": t_imul, "t_generator_ms": t_gen})
@@ -768,7 +781,8 @@ def run_sweep(args, rank, world, dist):
                           rewards="N(0,1) used as the normalised rewards; paper-scale coefficients"),
            "peaks": {"hbm_gbs": hbm_gbs, "hbm_source": peak_src,
                      "imul32_per_s": imul_peak, "gauss_per_s_imul": gauss_peak,
-                     "gauss_per_s_generator": gen_peak, "sms": sms,
+                     "gauss_per_s_generator": gen_peak,
+                     "gauss_per_s_generator_pipelined": gen_pipe, "sms": sms,
                      "sm_max_mhz": sm_max_mhz},
            "bytes_per_launch": bytes_per_launch, "points": points,
            "gpu_launches": launches, "clocks": clk.summary()}

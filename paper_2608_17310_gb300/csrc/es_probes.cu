@@ -56,6 +56,7 @@ enum Probe : int {
   kPhilox,
   kGenerator,
   kImadWideMul,
+  kGeneratorPipelined,
   kProbeCount
 };
 
@@ -89,9 +90,12 @@ const ProbeInfo kInfo[kProbeCount] = {
     {"split_imad_wide_only", "mad.wide.u32 (even warps; odd warps idle)", 8, 0.5},
     {"split_mufu_only", "MUFU (odd warps; even warps idle)", 16.0 / kSplitMufuDiv, 0.5},
     {"split_both", "warp-iterations (even warps mad.wide, odd warps MUFU)", 1, 1},
-    {"philox", "Philox4x32-10 block", 2, 1},
+    {"philox", "Philox4x32-10 block (round keys from the launch's parameters)", 2, 1},
     {"generator", "Gaussian (Philox4x32-10 + Box-Muller)", 8, 1},
     {"imad_wide_mul", "mul.wide.u32 by a constant (no addend), with one add each", 8, 1},
+    {"generator_pipelined",
+     "Gaussian (two seeds alternating, the next one's Philox beside the current transform)", 16,
+     1},
 };
 
 __device__ __forceinline__ uint64_t mad_wide(uint32_t a, uint64_t c) {
@@ -128,10 +132,17 @@ __device__ __forceinline__ float mufu2(float a) {
   return e;
 }
 
+// Round-key schedules of two seeds, passed as a __grid_constant__ parameter as
+// the perturb/restore kernels pass theirs: every round key is a constant-bank
+// operand, so the generator probes run the kernels' instruction stream.
+struct ProbeKeys {
+  esopt::PhiloxSched s[2];
+};
+
 template <int P>
 __global__ void __launch_bounds__(kThreads)
 probe_kernel(int iters, uint32_t seed, unsigned long long* __restrict__ rec,
-             uint32_t* __restrict__ sink) {
+             uint32_t* __restrict__ sink, const __grid_constant__ ProbeKeys keys) {
   const uint32_t t = seed + threadIdx.x * 0x9E3779B9u + blockIdx.x;
   uint64_t w[9];
   uint32_t x[8], y[8];
@@ -268,12 +279,14 @@ probe_kernel(int iters, uint32_t seed, unsigned long long* __restrict__ rec,
       m[1] = mufu2(m[1]);
     }
   } else if constexpr (P == kPhilox) {
-    const esopt::PhiloxTile pt = esopt::philox_tile(0u, esopt::philox_key(seed));
+    // the kernels' Philox alone: round keys from the launch's parameters
+    const esopt::PhiloxSched& ps = keys.s[0];
+    const esopt::TileConst tc = esopt::tile_const(0u, ps.rk[0], ps.rk[3]);
     uint32_t j = t * 2u;
 #pragma unroll 1
     for (int i = 0; i < iters; ++i) {
-      const uint4 a = esopt::philox_block_tile(j, pt);
-      const uint4 b = esopt::philox_block_tile(j + 1u, pt);
+      const uint4 a = esopt::philox_block_rk<false>(j, tc, ps.rk[1], ps.rk[2], ps.rk + 4);
+      const uint4 b = esopt::philox_block_rk<false>(j + 1u, tc, ps.rk[1], ps.rk[2], ps.rk + 4);
       x[0] ^= a.x ^ b.x;
       x[1] ^= a.y ^ b.y;
       x[2] ^= a.z ^ b.z;
@@ -294,10 +307,10 @@ probe_kernel(int iters, uint32_t seed, unsigned long long* __restrict__ rec,
         y[k] += lo;
       }
   } else if constexpr (P == kGenerator) {
-    // the kernels' generator: round keys from a precomputed schedule, the
+    // the kernels' generator: round keys from the launch's parameters, the
     // packed transform from the hardware log2, the near-one series on a rare
     // branch, then the square roots
-    const esopt::PhiloxSched ps = esopt::philox_sched(seed);
+    const esopt::PhiloxSched& ps = keys.s[0];
     const esopt::TileConst tc = esopt::tile_const(0u, ps.rk[0], ps.rk[3]);
     uint32_t j = t * 2u;
     float2 s0 = make_float2(0.f, 0.f), s1 = s0;
@@ -321,6 +334,49 @@ probe_kernel(int iters, uint32_t seed, unsigned long long* __restrict__ rec,
       j += 0x20000u;
     }
     f[0] = s0.x + s0.y + s1.x + s1.y;
+  } else if constexpr (P == kGeneratorPipelined) {
+    // the update's seed loop in registers: the blocks of two seeds alternate,
+    // and the next seed's Philox words are computed in the same basic block
+    // as the current seed's transform, on alternating word buffers
+    const esopt::PhiloxSched& ps0 = keys.s[0];
+    const esopt::PhiloxSched& ps1 = keys.s[1];
+    const esopt::TileConst tc0 = esopt::tile_const(0u, ps0.rk[0], ps0.rk[3]);
+    const esopt::TileConst tc1 = esopt::tile_const(0u, ps1.rk[0], ps1.rk[3]);
+    uint32_t j = t * 2u;
+    float2 s0 = make_float2(0.f, 0.f), s1 = s0;
+    auto words = [&](const esopt::PhiloxSched& ps, const esopt::TileConst& tc, uint32_t jj,
+                     uint4 (&x)[2]) {
+#pragma unroll
+      for (int b = 0; b < 2; ++b)
+        x[b] = esopt::philox_block_rk<false>(jj + b, tc, ps.rk[1], ps.rk[2], ps.rk + 4);
+    };
+    auto transform = [&](const uint4 (&x)[2]) {
+      uint2 xa[2];
+      esopt::Polar2 p[2];
+#pragma unroll
+      for (int b = 0; b < 2; ++b) {
+        xa[b] = make_uint2(x[b].x, x[b].z);
+        p[b] = esopt::polar2_sq<true>(x[b]);
+      }
+      esopt::fix_near_one<2>(xa, p);
+#pragma unroll
+      for (int b = 0; b < 2; ++b) {
+        const float2 r = make_float2(esopt::sqrt_approx(p[b].r.x), esopt::sqrt_approx(p[b].r.y));
+        s0 = __ffma2_rn(make_float2(r.x, r.x), make_float2(p[b].c.x, p[b].s.x), s0);
+        s1 = __ffma2_rn(make_float2(r.y, r.y), make_float2(p[b].c.y, p[b].s.y), s1);
+      }
+    };
+    uint4 xa0[2], xb0[2];
+    words(ps0, tc0, j, xa0);
+#pragma unroll 1
+    for (int i = 0; i < iters; ++i) {
+      words(ps1, tc1, j, xb0);
+      transform(xa0);
+      j += 0x20000u;
+      words(ps0, tc0, j, xa0);
+      transform(xb0);
+    }
+    f[0] = s0.x + s0.y + s1.x + s1.y + __uint_as_float(xa0[0].x & 0x3F000000u);
   }
 
   __syncthreads();
@@ -358,7 +414,7 @@ void* const kKernels[kProbeCount] = {
     kernel_of<4>(),  kernel_of<5>(),  kernel_of<6>(),  kernel_of<7>(),
     kernel_of<8>(),  kernel_of<9>(),  kernel_of<10>(), kernel_of<11>(),
     kernel_of<12>(), kernel_of<13>(), kernel_of<14>(), kernel_of<15>(),
-    kernel_of<16>(), kernel_of<17>(), kernel_of<18>(),
+    kernel_of<16>(), kernel_of<17>(), kernel_of<18>(), kernel_of<19>(),
 };
 
 }  // namespace
@@ -408,11 +464,14 @@ int esprobe_run(int probe, int ctas_per_sm, int iters, double* out) {
   float ms = 0.0f;
   if (err == cudaSuccess) {
     uint32_t seed = 0x51ED270Bu;
+    ProbeKeys keys;
+    keys.s[0] = esopt::philox_sched(seed);
+    keys.s[1] = esopt::philox_sched(seed + 1u);
     int warm_iters = iters / 8 > 0 ? iters / 8 : 1;
-    void* warm[] = {&warm_iters, &seed, &rec, &sink};
+    void* warm[] = {&warm_iters, &seed, &rec, &sink, &keys};
     err = cudaLaunchKernel(kKernels[probe], dim3(grid), dim3(kThreads), warm, 0, 0);
     if (err == cudaSuccess) err = cudaEventRecord(e0, 0);
-    void* args[] = {&iters, &seed, &rec, &sink};
+    void* args[] = {&iters, &seed, &rec, &sink, &keys};
     if (err == cudaSuccess)
       err = cudaLaunchKernel(kKernels[probe], dim3(grid), dim3(kThreads), args, 0, 0);
     if (err == cudaSuccess) err = cudaEventRecord(e1, 0);
