@@ -57,6 +57,7 @@ enum Probe : int {
   kGenerator,
   kImadWideMul,
   kGeneratorPipelined,
+  kGeneratorSplit,
   kProbeCount
 };
 
@@ -96,7 +97,45 @@ const ProbeInfo kInfo[kProbeCount] = {
     {"generator_pipelined",
      "Gaussian (two seeds alternating, the next one's Philox beside the current transform)", 16,
      1},
+    {"generator_split",
+     "Gaussian (Philox on warps 0-3, Box-Muller on warps 4-7, warp pairs through shared memory)",
+     8, 0.5},
 };
+
+// Shared-memory slots of the split generator probe, and the most polls of an
+// mbarrier before a wait gives up (the probe then stops and reports it).
+constexpr int kSplitStages = 8;
+constexpr int kWaitPolls = 1 << 20;
+
+__device__ __forceinline__ uint32_t smem_u32(const void* p) {
+  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+__device__ __forceinline__ void mbar_init(uint64_t* bar, uint32_t count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)), "r"(count)
+               : "memory");
+}
+__device__ __forceinline__ void mbar_arrive(uint64_t* bar) {
+  uint64_t state;
+  asm volatile("mbarrier.arrive.shared::cta.b64 %0, [%1];"
+               : "=l"(state)
+               : "r"(smem_u32(bar))
+               : "memory");
+}
+// Waits for the completion of the barrier's phase of the given parity; false
+// if it has not completed after kWaitPolls polls.
+__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity) {
+  for (int n = 0; n < kWaitPolls; ++n) {
+    uint32_t done;
+    asm volatile(
+        "{\n\t.reg .pred p;\n\tmbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}"
+        : "=r"(done)
+        : "r"(smem_u32(bar)), "r"(parity)
+        : "memory");
+    if (done) return true;
+  }
+  return false;
+}
 
 __device__ __forceinline__ uint64_t mad_wide(uint32_t a, uint64_t c) {
   uint64_t d;
@@ -377,6 +416,70 @@ probe_kernel(int iters, uint32_t seed, unsigned long long* __restrict__ rec,
       transform(xb0);
     }
     f[0] = s0.x + s0.y + s1.x + s1.y + __uint_as_float(xa0[0].x & 0x3F000000u);
+  } else if constexpr (P == kGeneratorSplit) {
+    // Philox and Box-Muller on separate warps: producer warp w (0-3) writes
+    // the words of two blocks per thread and iteration into its own ring of
+    // kSplitStages shared slots, consumer warp w + 4 transforms them. Each
+    // slot of a pair is handed over by mbarriers of 32 arrivals: full when
+    // the producer warp has written it, empty when the consumer warp has read
+    // it. Both warps of a pair run the same iterations in the same slot
+    // order; every wait is bounded, and a thread whose wait gives up stops
+    // (its partner's waits then give up too) and flags it in sink[1].
+    __shared__ uint4 ring[kSplitStages][4][32][2];
+    __shared__ uint64_t full_bar[kSplitStages][4], empty_bar[kSplitStages][4];
+    if (threadIdx.x < 4 * kSplitStages) {
+      mbar_init(&full_bar[threadIdx.x / 4][threadIdx.x % 4], 32);
+      mbar_init(&empty_bar[threadIdx.x / 4][threadIdx.x % 4], 32);
+    }
+    __syncthreads();
+    const int pair = (threadIdx.x >> 5) & 3, lane = threadIdx.x & 31;
+    bool ok = true;
+    if (threadIdx.x < 128) {
+      const esopt::PhiloxSched& ps = keys.s[0];
+      const esopt::TileConst tc = esopt::tile_const(0u, ps.rk[0], ps.rk[3]);
+      uint32_t j = t * 2u;
+#pragma unroll 1
+      for (int i = 0; i < iters; ++i) {
+        const int st = i % kSplitStages;
+        const uint32_t use = static_cast<uint32_t>(i / kSplitStages);
+        if (use > 0 && !mbar_wait(&empty_bar[st][pair], (use - 1) & 1u)) {
+          ok = false;
+          break;
+        }
+        ring[st][pair][lane][0] =
+            esopt::philox_block_rk<false>(j, tc, ps.rk[1], ps.rk[2], ps.rk + 4);
+        ring[st][pair][lane][1] =
+            esopt::philox_block_rk<false>(j + 1u, tc, ps.rk[1], ps.rk[2], ps.rk + 4);
+        mbar_arrive(&full_bar[st][pair]);
+        j += 0x20000u;
+      }
+    } else {
+      float2 s0 = make_float2(0.f, 0.f), s1 = s0;
+#pragma unroll 1
+      for (int i = 0; i < iters; ++i) {
+        const int st = i % kSplitStages;
+        const uint32_t use = static_cast<uint32_t>(i / kSplitStages);
+        if (!mbar_wait(&full_bar[st][pair], use & 1u)) {
+          ok = false;
+          break;
+        }
+        const uint4 x0 = ring[st][pair][lane][0], x1 = ring[st][pair][lane][1];
+        // the slot is free again; its last use needs no release
+        if (i + kSplitStages < iters) mbar_arrive(&empty_bar[st][pair]);
+        uint2 xa[2] = {make_uint2(x0.x, x0.z), make_uint2(x1.x, x1.z)};
+        esopt::Polar2 p[2] = {esopt::polar2_sq<true>(x0), esopt::polar2_sq<true>(x1)};
+        esopt::fix_near_one<2>(xa, p);
+#pragma unroll
+        for (int b = 0; b < 2; ++b) {
+          const float2 r =
+              make_float2(esopt::sqrt_approx(p[b].r.x), esopt::sqrt_approx(p[b].r.y));
+          s0 = __ffma2_rn(make_float2(r.x, r.x), make_float2(p[b].c.x, p[b].s.x), s0);
+          s1 = __ffma2_rn(make_float2(r.y, r.y), make_float2(p[b].c.y, p[b].s.y), s1);
+        }
+      }
+      f[0] = s0.x + s0.y + s1.x + s1.y;
+    }
+    if (!ok) sink[1] = 1u;
   }
 
   __syncthreads();
@@ -415,6 +518,7 @@ void* const kKernels[kProbeCount] = {
     kernel_of<8>(),  kernel_of<9>(),  kernel_of<10>(), kernel_of<11>(),
     kernel_of<12>(), kernel_of<13>(), kernel_of<14>(), kernel_of<15>(),
     kernel_of<16>(), kernel_of<17>(), kernel_of<18>(), kernel_of<19>(),
+    kernel_of<20>(),
 };
 
 }  // namespace
@@ -440,7 +544,8 @@ const char* esprobe_unit(int probe) {
 // out[0..6] = milliseconds (CUDA events), mean SM cycles per SM (that span),
 // SM clock in MHz (CTA cycles / globaltimer ns), ops per clock per SM, ops in
 // total, active threads per SM, CTAs per SM used. Returns 0, -1 for a bad
-// argument, else the cudaError_t.
+// argument, -2 if a bounded wait of the split probe gave up, else the
+// cudaError_t.
 int esprobe_run(int probe, int ctas_per_sm, int iters, double* out) {
   if (probe < 0 || probe >= kProbeCount || ctas_per_sm < 1 || iters < 1 || out == nullptr)
     return -1;
@@ -457,11 +562,13 @@ int esprobe_run(int probe, int ctas_per_sm, int iters, double* out) {
   uint32_t* sink = nullptr;
   cudaEvent_t e0 = nullptr, e1 = nullptr;
   err = cudaMalloc(&rec, sizeof(unsigned long long) * 4 * grid);
-  if (err == cudaSuccess) err = cudaMalloc(&sink, sizeof(uint32_t));
+  if (err == cudaSuccess) err = cudaMalloc(&sink, 2 * sizeof(uint32_t));
+  if (err == cudaSuccess) err = cudaMemset(sink, 0, 2 * sizeof(uint32_t));
   if (err == cudaSuccess) err = cudaEventCreate(&e0);
   if (err == cudaSuccess) err = cudaEventCreate(&e1);
   unsigned long long* host = new unsigned long long[4 * grid];
   float ms = 0.0f;
+  bool waits_gave_up = false;
   if (err == cudaSuccess) {
     uint32_t seed = 0x51ED270Bu;
     ProbeKeys keys;
@@ -479,6 +586,10 @@ int esprobe_run(int probe, int ctas_per_sm, int iters, double* out) {
     if (err == cudaSuccess) err = cudaEventElapsedTime(&ms, e0, e1);
     if (err == cudaSuccess)
       err = cudaMemcpy(host, rec, sizeof(unsigned long long) * 4 * grid, cudaMemcpyDeviceToHost);
+    uint32_t gave_up = 0;
+    if (err == cudaSuccess)
+      err = cudaMemcpy(&gave_up, sink + 1, sizeof(uint32_t), cudaMemcpyDeviceToHost);
+    if (err == cudaSuccess && gave_up != 0) waits_gave_up = true;
   }
   if (err == cudaSuccess) {
     // per SM: [first start, last end] on its own clock (%smid may exceed the
@@ -527,6 +638,7 @@ int esprobe_run(int probe, int ctas_per_sm, int iters, double* out) {
   if (e1) cudaEventDestroy(e1);
   cudaFree(rec);
   cudaFree(sink);
+  if (err == cudaSuccess && waits_gave_up) return -2;
   return static_cast<int>(err);
 }
 
