@@ -76,6 +76,16 @@ constexpr int kVecsPerThread = ES_VECS_PER_THREAD;
 #ifndef ES_UPDATE_PIPELINED
 #define ES_UPDATE_PIPELINED 2
 #endif
+// The antithetic flip (es_restore_perturb with one seed) in the scalar form
+// per block (0) or in the packed form of the other passes, with round 0's
+// product stepped in tiles inside their segment (1); values identical. Its
+// resident CTAs per SM (a register cap), like the other passes'.
+#ifndef ES_FLIP_PACKED
+#define ES_FLIP_PACKED 1
+#endif
+#ifndef ES_FLIP_MIN_BLOCKS
+#define ES_FLIP_MIN_BLOCKS 3
+#endif
 // Round 0's Philox product (kPhiloxMulA times the low counter word) depends
 // on the counter alone: 0 computes it per block and seed; 1 once per block,
 // shared by the seeds of a pass (both seeds of the fused restore + perturb,
@@ -98,10 +108,9 @@ constexpr int kUpdateGroup = ES_UPDATE_GROUP;
 static_assert(kVecsPerThread % kAxpy1Group == 0 && kVecsPerThread % kAxpy2Group == 0 &&
                   kVecsPerThread % kUpdateGroup == 0,
               "groups divide the vectors of a tile");
-constexpr int axpy_min_blocks(bool two, int vec_elems = 8) {
-  const int m = (two ? ES_AXPY2_MIN_BLOCKS : ES_AXPY1_MIN_BLOCKS) > 0
-                    ? (two ? ES_AXPY2_MIN_BLOCKS : ES_AXPY1_MIN_BLOCKS)
-                    : 1;
+constexpr int axpy_min_blocks(bool two, int vec_elems = 8, bool same = false) {
+  const int want = same ? ES_FLIP_MIN_BLOCKS : two ? ES_AXPY2_MIN_BLOCKS : ES_AXPY1_MIN_BLOCKS;
+  const int m = want > 0 ? want : 1;
   // FP8 vectors hold twice the elements (twice the Philox blocks per vector):
   // at most 2 CTAs per SM, so their registers do not spill
   return vec_elems > 8 && m > 2 ? 2 : m;

@@ -218,6 +218,7 @@ constexpr NoiseForm kUpdateForm = static_cast<NoiseForm>(ES_UPDATE_FORM);
 constexpr bool kUpdatePipelined = ES_UPDATE_PIPELINED != 0;
 constexpr bool kUpdatePingPong = ES_UPDATE_PIPELINED >= 2;
 constexpr int kRound0 = ES_ROUND0;
+constexpr bool kFlipPacked = ES_FLIP_PACKED != 0;
 // Near-one radius inputs: a rare branch (true) or a select per pair (false).
 constexpr bool kNearOneBranch = ES_NEAR_ONE_BRANCH != 0;
 
@@ -442,7 +443,9 @@ __device__ __forceinline__ void axpy_tile(const TileRef<Io>& cur, uint4 (&v)[G],
   // from the thread's first block (its blocks share the high counter word,
   // so j_lo + d never wraps).
   constexpr int NB = V / 4;
-  constexpr bool kR0 = kUniformHi && !kSame && (kRound0 >= 2 ? (kFull || kTwo) : kRound0 >= 1 && kTwo);
+  constexpr bool kR0 = kUniformHi && (kSame ? kFlipPacked && kFull && kRound0 >= 2
+                                            : (kRound0 >= 2 ? (kFull || kTwo)
+                                                            : kRound0 >= 1 && kTwo));
   constexpr bool kR0Step = kR0 && kFull && kRound0 >= 2;
   Round0 p0_thread{0u, 0u};
   if constexpr (kR0Step) p0_thread = philox_round0<kWide1>(static_cast<uint32_t>(j_thread));
@@ -470,7 +473,23 @@ __device__ __forceinline__ void axpy_tile(const TileRef<Io>& cur, uint4 (&v)[G],
       const uint64_t j0 = j_thread + static_cast<uint64_t>(u) * (kStride / 4);
       float f[V];
       Io::unpack(v[q], f);
-      if constexpr (kSame) {
+      if constexpr (kSame && kFlipPacked) {
+        // one seed's noise for both steps, in the packed form
+        uint4 x[NB];
+        if constexpr (kR0) {
+#pragma unroll
+          for (int b = 0; b < NB; ++b)
+            x[b] = gen.block_r0(
+                round0_step(p0_thread, static_cast<uint32_t>(u * (kStride / 4) + b)));
+        } else {
+          philox_words<NB>(gen, j0, x);
+        }
+        Polar2 pp[NB];
+        polar_from_words<kAxpyForm, NB>(x, pp);
+        apply_noise<kAxpyForm, V>(pp, s1, f);
+        Io::round_trip(f);
+        apply_noise<kAxpyForm, V>(pp, s2, f);
+      } else if constexpr (kSame) {
         add_scaled_noise_twice<Io, V>(gen, j0, s1, s2, f);
       } else if constexpr (kR0) {
         Round0 p0[NB];
@@ -515,7 +534,7 @@ __device__ __forceinline__ void axpy_tile(const TileRef<Io>& cur, uint4 (&v)[G],
 // For a scaled storage type (FP8) the noise is added in units of the
 // segment's scale: scale * inv_scale[segment].
 template <class Io, bool kTwo, bool kSame>
-__global__ void __launch_bounds__(kBlockThreads, axpy_min_blocks(kTwo, Io::kVec))
+__global__ void __launch_bounds__(kBlockThreads, axpy_min_blocks(kTwo, Io::kVec, kSame))
 axpy_noise_kernel(const SegDesc* __restrict__ segs, const float* __restrict__ inv_scale,
                   uint64_t total_tiles, const __grid_constant__ AxpyArgs a) {
   constexpr int G = group_for<Io>(kTwo ? kAxpy2Group : kAxpy1Group);
