@@ -820,3 +820,65 @@ def test_near_one_radius_inputs_match_oracle(es, oracle, dtype):
                 noise_abs_tol([oracle.noise_at(s2, sel2), oracle.noise_at(s, sel2)],
                               [coeffs[0], sigma]))
     plan.close()
+
+
+@pytest.mark.parametrize("dtype", ["bf16", "f32"])
+def test_tiles_meeting_a_high_counter_word_boundary(es, oracle, dtype):
+    # Inside a tile whose blocks share the high counter word, the kernels take
+    # round 0's Philox product of a thread's later blocks from its first one's
+    # by 64-bit additions, which is exact only while the low counter word does
+    # not wrap. Here three whole tiles end exactly at block 2^32 (their last
+    # low word is 2^32 - 1) and three more start there, plus a ragged tail;
+    # every call is checked on every element: against the oracle one step at a
+    # time, and the fused calls bit for bit against the separate ones.
+    tile = 256 * 4 * (8 if dtype == "bf16" else 4)
+    n = 6 * tile + 5
+    a = make_params(dtype, [n], seed=21)
+    b = [t.clone() for t in a]
+    base = [2**34 - 3 * tile]
+    plan_a, segs = build_plan(es, a, base)
+    plan_b, _ = build_plan(es, b, base)
+    g = indices(segs)[0]
+    iv = torch.int16 if dtype == "bf16" else torch.int32
+    s1, s2, sig = 2**40 + 3, 77, 1e-3
+
+    before = host_values(a[0])
+    for p in (plan_a, plan_b):
+        es.es_perturb(p, s1, sig)
+    torch.cuda.synchronize()
+    got = host_values(a[0])
+    compare(dtype, got, oracle.perturb(before, g, s1, sig, dtype), "perturb",
+            noise_abs_tol([oracle.noise_at(s1, g)], [sig]))
+    # fused restore + perturb against the two separate calls, each checked
+    es.es_restore_perturb(plan_a, s1, sig, s2, sig)
+    es.es_restore(plan_b, s1, sig)
+    torch.cuda.synchronize()
+    mid = host_values(b[0])
+    compare(dtype, mid, oracle.restore(got, g, s1, sig, dtype), "restore",
+            noise_abs_tol([oracle.noise_at(s1, g)], [sig]))
+    es.es_perturb(plan_b, s2, sig)
+    torch.cuda.synchronize()
+    assert torch.equal(a[0].view(iv), b[0].view(iv))
+    compare(dtype, host_values(b[0]), oracle.perturb(mid, g, s2, sig, dtype), "perturb 2",
+            noise_abs_tol([oracle.noise_at(s2, g)], [sig]))
+    # the antithetic flip against the separate restore and perturb with -sigma
+    es.es_restore_perturb(plan_a, s2, sig, s2, -sig)
+    es.es_restore(plan_b, s2, sig)
+    es.es_perturb(plan_b, s2, -sig)
+    torch.cuda.synchronize()
+    assert torch.equal(a[0].view(iv), b[0].view(iv))
+    # the update (and its fused perturb) on the same tiles
+    seeds = np.array([5, 2**33 + 1, 99], dtype=np.uint64)
+    coeffs = np.array([1e-3, -2e-3, 5e-4], dtype=np.float32)
+    before = host_values(a[0])
+    es.es_update_perturb(plan_a, seeds, coeffs, s1, sig)
+    es.es_update(plan_b, seeds, coeffs)
+    torch.cuda.synchronize()
+    upd = host_values(b[0])
+    compare(dtype, upd, oracle.update(before, g, seeds, coeffs, dtype), "update",
+            noise_abs_tol([oracle.noise_at(int(s), g) for s in seeds], coeffs))
+    es.es_perturb(plan_b, s1, sig)
+    torch.cuda.synchronize()
+    assert torch.equal(a[0].view(iv), b[0].view(iv))
+    plan_a.close()
+    plan_b.close()
